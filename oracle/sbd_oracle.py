@@ -1,0 +1,239 @@
+"""fp64 CPU oracle for the Set Block Decoding (SBD) block step.
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, the smoke check of the graft entry
+point and the CPU-baseline leg of the bench may import or call this module.
+The product path (the CUDA library and its Python binding) never does, and it
+shares no code with it: this file imports numpy and nothing else of the repo.
+
+Every function is the plain definition written out in float64 over the input
+values (bf16 inputs are widened exactly), with library primitives (matmul,
+exp, log, sort) as the only helpers and no blocking or fusion beyond what the
+definition states.  Each cites the passage of arXiv 2509.04185 it follows.
+
+Readings of points the paper leaves open (each listed in the design notes):
+  * softmax scale 1/sqrt(head_dim) unless given;
+  * grouped-query heads: query head hq reads KV head hq // (Hq / Hkv);
+  * entropy in nats of softmax(z) at temperature 1;
+  * sampling is Gumbel-max on z + tau * g (tau = 0: greedy, the paper's
+    temperature-0 setting), ties to the lowest vocabulary id;
+  * EB rule with the inequality exactly as printed (<=), gamma = 0 allowed,
+    equal entropies ordered by block position.
+
+Pins (what each function is checked against, none of it itself) live in
+tests/test_oracle_*.py; no function here is "parity unpinned".
+"""
+from __future__ import annotations
+
+import numpy as np
+
+MASK_TOKEN = -1
+
+
+# ----------------------------------------------------------------- inputs
+
+def widen(x: np.ndarray, dtype: str) -> np.ndarray:
+    """Storage -> float64.  bf16 is stored as its raw 16-bit pattern, which is
+    the upper half of the fp32 with the same value, so widening is exact."""
+    if dtype == "bf16":
+        bits = np.asarray(x, dtype=np.uint16).astype(np.uint32) << 16
+        return bits.view(np.float32).astype(np.float64)
+    if dtype == "f32":
+        return np.asarray(x, dtype=np.float32).astype(np.float64)
+    return np.asarray(x, dtype=np.float64)
+
+
+# ------------------------------------------------------------- attention
+
+def inference_mask_allows(q_idx: int, kv_idx: int, causal_point: int) -> bool:
+    """Inference attention mask of the SBD network (Eq. 5 and the inference
+    mask of the FlexAttention appendix): a query may see a key when the key is
+    not in its future, or when the query lies in the prediction block, which
+    starts at causal_point; block queries therefore see every key."""
+    return (kv_idx <= q_idx) or (causal_point <= q_idx)
+
+
+def block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None):
+    """Block attention of one SBD forward (Eq. 5; Fig. 3 mask).
+
+    Block query row i of sequence b attends to the L_b cached keys (the exact
+    KV cache of x_<t, causal among themselves and all in the past of the
+    block) and to all k block keys (bidirectional inside the block).
+
+    q [B,k,Hq,D]; k_cache, v_cache [B,Lmax,Hkv,D]; cache_len [B];
+    k_blk, v_blk [B,k,Hkv,D]; all float64.  Returns o [B,k,Hq,D] float64.
+    """
+    B, k, Hq, D = q.shape
+    Hkv = k_cache.shape[2]
+    G = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    out = np.zeros((B, k, Hq, D), dtype=np.float64)
+    for b in range(B):
+        L = int(cache_len[b])
+        for hq in range(Hq):
+            hk = hq // G
+            keys = np.concatenate([k_cache[b, :L, hk, :], k_blk[b, :, hk, :]], axis=0)
+            vals = np.concatenate([v_cache[b, :L, hk, :], v_blk[b, :, hk, :]], axis=0)
+            s = (q[b, :, hq, :] @ keys.T) * scale            # [k, L+k]
+            s = s - s.max(axis=1, keepdims=True)
+            p = np.exp(s)
+            p = p / p.sum(axis=1, keepdims=True)
+            out[b, :, hq, :] = p @ vals
+    return out
+
+
+def masked_sequence_attention(q_seq, k_seq, v_seq, causal_point, scale=None):
+    """Brute force: full-sequence attention under the explicit inference mask
+    predicate, for one head.  q_seq, k_seq, v_seq [T, D].  Used only to pin
+    block_attention on tiny inputs."""
+    T, D = q_seq.shape
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    out = np.zeros((T, D), dtype=np.float64)
+    for qi in range(T):
+        allowed = [j for j in range(T) if inference_mask_allows(qi, j, causal_point)]
+        s = np.array([float(q_seq[qi] @ k_seq[j]) * scale for j in allowed])
+        s = s - s.max()
+        p = np.exp(s)
+        p = p / p.sum()
+        out[qi] = sum(p[a] * v_seq[j] for a, j in enumerate(allowed))
+    return out
+
+
+# ------------------------------------------------------------- LM head
+
+def logits(hidden_rows: np.ndarray, w_store: np.ndarray, w_dtype: str,
+           vocab_chunk: int = 8192) -> np.ndarray:
+    """z_{r,v} = sum_c h_{r,c} W_{v,c}: the LM head that produces the block
+    logits z_hat of Eq. 5 (nn.Linear layout, W [V,H]).  hidden_rows [R,H]
+    float64; w_store [V,H] in storage form.  Vocabulary rows are widened one
+    slice at a time only to bound memory: every logit is the same single dot
+    product."""
+    R = hidden_rows.shape[0]
+    V = w_store.shape[0]
+    z = np.empty((R, V), dtype=np.float64)
+    for v0 in range(0, V, vocab_chunk):
+        v1 = min(V, v0 + vocab_chunk)
+        z[:, v0:v1] = hidden_rows @ widen(w_store[v0:v1], w_dtype).T
+    return z
+
+
+def entropy(z_row: np.ndarray) -> float:
+    """H(p) = -sum_v p_v log p_v in nats, p = softmax(z) (the entropy of the
+    predicted marginal used by the EB rule, Eq. 3); 0 log 0 := 0.  Computed
+    with the max subtracted for range: log p_v = (z_v - max z) - log Z."""
+    z = np.asarray(z_row, dtype=np.float64)
+    m = z.max()
+    e = np.exp(z - m)
+    Z = e.sum()
+    p = e / Z
+    logp = (z - m) - np.log(Z)
+    terms = np.where(p > 0.0, -p * logp, 0.0)
+    return float(terms.sum())
+
+
+def sample_token(z_row: np.ndarray, g_row, tau: float) -> int:
+    """Gumbel-max sample: argmax_v (z_v + tau * g_v); tau = 0 (or no noise)
+    is greedy decoding, the paper's temperature-0 setting (Sec. 3.1).  For
+    tau > 0 this samples softmax(z / tau).  Ties go to the lowest id."""
+    z = np.asarray(z_row, dtype=np.float64)
+    if tau == 0.0 or g_row is None:
+        score = z
+    else:
+        score = z + float(tau) * np.asarray(g_row, dtype=np.float64)
+    return int(np.argmax(score))          # first maximum = lowest id
+
+
+def head_entropy_sample(hidden, w_store, w_dtype, masked, gumbel, tau,
+                        rows=None, vocab_chunk: int = 8192):
+    """Per block position: entropy (nats) and sampled token of the masked
+    positions' predicted marginals p_theta(x_{t+i} | x_<t; x_hat) (Eqs. 6-7,
+    Algorithm 3 "compute probabilities").  Position t+i predicts its own
+    token (no shift).
+
+    hidden [B,k,H] float64; w_store [V,H] storage; masked [B,k] (nonzero =
+    masked); gumbel [B,k,V] or None.  Unmasked positions get entropy +inf and
+    token -1.  `rows`, if given, restricts the work to those (b, i) pairs
+    (the others are left as +inf / -1).  Returns (entropy [B,k] f64,
+    token [B,k] int32, z dict {(b,i): z_row}) -- z is returned for test
+    diagnostics (top-2 gaps)."""
+    B, k, H = hidden.shape
+    ent = np.full((B, k), np.inf, dtype=np.float64)
+    tok = np.full((B, k), MASK_TOKEN, dtype=np.int32)
+    if rows is None:
+        rows = [(b, i) for b in range(B) for i in range(k) if masked[b, i]]
+    else:
+        rows = [(b, i) for (b, i) in rows if masked[b, i]]
+    if not rows:
+        return ent, tok, {}
+    hr = np.stack([hidden[b, i] for (b, i) in rows])
+    z = logits(hr, w_store, w_dtype, vocab_chunk)
+    zs = {}
+    for n, (b, i) in enumerate(rows):
+        ent[b, i] = entropy(z[n])
+        g = None if gumbel is None else gumbel[b, i]
+        tok[b, i] = sample_token(z[n], g, tau)
+        zs[(b, i)] = z[n]
+    return ent, tok, zs
+
+
+# ------------------------------------------------------------- EB select
+
+def eb_accept_count(sorted_entropies, gamma: float) -> int:
+    """EB-Sampler, entropy proxy (Eq. 3): with the masked entropies sorted
+    ascending, s >= 1 is the largest integer with
+        sum_{j=1}^{s-1} H_{i_j} <= gamma,
+    capped at |M|.  Prefix sums in float64.  For non-negative entropies the
+    prefix sums are non-decreasing, so the largest such s is found by walking
+    the sorted list until the first prefix sum above gamma."""
+    n = len(sorted_entropies)
+    if n == 0:
+        return 0
+    s = 1
+    prefix = 0.0
+    for j in range(1, n):                  # candidate s = j + 1 needs S_j
+        prefix += float(sorted_entropies[j - 1])
+        if prefix <= gamma:
+            s = j + 1
+        else:
+            break
+    return s
+
+
+def eb_select(entropy_bk, token_bk, masked_bk, block_tokens_bk, gamma: float):
+    """One EB unmasking step over a batch (Algorithm 3, "unmask tokens
+    according to Eq. 3").  Per sequence: sort the masked positions by
+    (entropy, position) ascending, accept the first s of Eq. 3, write their
+    sampled tokens into the block buffer and clear their masked flags.
+
+    Returns (new_masked [B,k] uint8, new_block_tokens [B,k] int32,
+    n_unmasked [B] int32, accepted list of sets, sorted orders)."""
+    B, k = masked_bk.shape
+    new_masked = np.array(masked_bk, dtype=np.uint8, copy=True)
+    new_bt = np.array(block_tokens_bk, dtype=np.int32, copy=True)
+    n_un = np.zeros(B, dtype=np.int32)
+    accepted = []
+    orders = []
+    for b in range(B):
+        M = [i for i in range(k) if masked_bk[b, i]]
+        order = sorted(M, key=lambda i: (float(entropy_bk[b, i]), i))
+        s = eb_accept_count([entropy_bk[b, i] for i in order], gamma)
+        acc = set(order[:s])
+        for i in acc:
+            new_bt[b, i] = token_bk[b, i]
+            new_masked[b, i] = 0
+        n_un[b] = s
+        accepted.append(acc)
+        orders.append(order)
+    return new_masked, new_bt, n_un, accepted, orders
+
+
+def eb_prefix_margins(entropy_row_sorted, gamma: float):
+    """|S_{j-1} - gamma| for each rank j >= 2 (1-based) of a sorted list:
+    the oracle's margin to gamma at each acceptance decision."""
+    out = []
+    prefix = 0.0
+    for j in range(1, len(entropy_row_sorted)):
+        prefix += float(entropy_row_sorted[j - 1])
+        out.append(abs(prefix - gamma))
+    return out

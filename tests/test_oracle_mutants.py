@@ -1,0 +1,176 @@
+"""Planted mistakes in the oracle must be caught by its pins (CPU only).
+
+Each mutant is the oracle with one plausible mistake (a dropped term, a wrong
+index, a wrong sign or inequality); the test runs the pins of the other
+oracle test files against it through monkeypatch and asserts that at least
+one of them fails."""
+import numpy as np
+import pytest
+
+import oracle
+import oracle.sbd_oracle as so
+from tests import test_oracle_attention as TA
+from tests import test_oracle_eb as TE
+from tests import test_oracle_head as TH
+
+
+def _fails(fn, *args):
+    try:
+        fn(*args)
+    except AssertionError:
+        return True
+    return False
+
+
+# ---------------------------------------------------------------- attention
+
+def _attn_drop_block(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None):
+    B, k, Hq, D = q.shape
+    G = Hq // k_cache.shape[2]
+    scale = 1.0 / np.sqrt(D) if scale is None else scale
+    out = np.zeros_like(q)
+    for b in range(B):
+        L = int(cache_len[b])
+        for hq in range(Hq):
+            hk = hq // G
+            keys = np.concatenate([k_cache[b, :L, hk], k_blk[b, :1, hk]])   # only one block key
+            vals = np.concatenate([v_cache[b, :L, hk], v_blk[b, :1, hk]])
+            s = q[b, :, hq] @ keys.T * scale
+            p = np.exp(s - s.max(axis=1, keepdims=True))
+            out[b, :, hq] = (p / p.sum(axis=1, keepdims=True)) @ vals
+    return out
+
+
+def _attn_mutant(scale_fn=None, head_fn=None):
+    def f(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None):
+        B, k, Hq, D = q.shape
+        Hkv = k_cache.shape[2]
+        G = Hq // Hkv
+        sc = (scale_fn(D) if scale_fn else 1.0 / np.sqrt(D)) if scale is None else scale
+        out = np.zeros_like(q)
+        for b in range(B):
+            L = int(cache_len[b])
+            for hq in range(Hq):
+                hk = head_fn(hq, G, Hkv) if head_fn else hq // G
+                keys = np.concatenate([k_cache[b, :L, hk], k_blk[b, :, hk]])
+                vals = np.concatenate([v_cache[b, :L, hk], v_blk[b, :, hk]])
+                s = q[b, :, hq] @ keys.T * sc
+                p = np.exp(s - s.max(axis=1, keepdims=True))
+                out[b, :, hq] = (p / p.sum(axis=1, keepdims=True)) @ vals
+        return out
+    return f
+
+
+ATTN_PINS = [
+    (TA.test_block_attention_equals_explicit_mask, (3, 4, 4, 2)),
+    (TA.test_k1_is_plain_causal_decode_sdpa, (8, 2)),
+    (TA.test_zero_query_is_uniform_average, ()),
+]
+
+
+@pytest.mark.parametrize("mutant", [
+    _attn_drop_block,
+    _attn_mutant(scale_fn=lambda D: 1.0 / D),
+    _attn_mutant(head_fn=lambda hq, G, Hkv: hq % Hkv),
+])
+def test_attention_mutants_are_caught(monkeypatch, mutant):
+    monkeypatch.setattr(oracle, "block_attention", mutant)
+    assert any(_fails(fn, *args) for fn, args in ATTN_PINS)
+
+
+# ---------------------------------------------------------------- entropy
+
+def _entropy_no_logz(z_row):
+    z = np.asarray(z_row, dtype=np.float64)
+    m = z.max()
+    e = np.exp(z - m)
+    p = e / e.sum()
+    return float((-p * (z - m)).sum())          # dropped the log Z term
+
+
+def _entropy_wrong_sign(z_row):
+    return -so.entropy(z_row)
+
+
+HEAD_PINS = [
+    (TH.test_uniform_logits_entropy_is_log_v, (512,)),
+    (TH.test_two_point_binary_entropy, (1.0, -0.5)),
+    (TH.test_entropy_matches_scipy_and_is_shift_invariant, ()),
+]
+
+
+@pytest.mark.parametrize("mutant", [_entropy_no_logz, _entropy_wrong_sign])
+def test_entropy_mutants_are_caught(monkeypatch, mutant):
+    monkeypatch.setattr(oracle, "entropy", mutant)
+    assert any(_fails(fn, *args) for fn, args in HEAD_PINS)
+
+
+def _token_ignores_tau(z_row, g_row, tau):
+    z = np.asarray(z_row, dtype=np.float64)
+    if g_row is None:
+        return int(np.argmax(z))
+    return int(np.argmax(z + np.asarray(g_row, dtype=np.float64)))
+
+
+def _token_last_tie(z_row, g_row, tau):
+    z = np.asarray(z_row, dtype=np.float64)
+    score = z if (tau == 0.0 or g_row is None) else z + tau * np.asarray(g_row)
+    return int(len(score) - 1 - np.argmax(score[::-1]))
+
+
+@pytest.mark.parametrize("mutant", [_token_ignores_tau, _token_last_tie])
+def test_token_mutants_are_caught(monkeypatch, mutant):
+    monkeypatch.setattr(oracle, "sample_token", mutant)
+    pins = [(TH.test_greedy_and_ties, ()), (TH.test_gumbel_max_is_softmax_sampling, (0.5,))]
+    assert any(_fails(fn, *args) for fn, args in pins)
+
+
+# ---------------------------------------------------------------- EB rule
+
+def _eb_strict(sorted_entropies, gamma):
+    n = len(sorted_entropies)
+    if n == 0:
+        return 0
+    s, prefix = 1, 0.0
+    for j in range(1, n):
+        prefix += float(sorted_entropies[j - 1])
+        if prefix < gamma:                     # < instead of <=
+            s = j + 1
+        else:
+            break
+    return s
+
+
+def _eb_includes_own(sorted_entropies, gamma):
+    n = len(sorted_entropies)
+    if n == 0:
+        return 0
+    s, prefix = 1, float(sorted_entropies[0])
+    for j in range(1, n):
+        prefix += float(sorted_entropies[j])   # S_s instead of S_{s-1}
+        if prefix <= gamma:
+            s = j + 1
+        else:
+            break
+    return s
+
+
+@pytest.mark.parametrize("mutant", [_eb_strict, _eb_includes_own])
+def test_eb_mutants_are_caught(monkeypatch, mutant):
+    monkeypatch.setattr(so, "eb_accept_count", mutant)
+    monkeypatch.setattr(oracle, "eb_accept_count", mutant)
+    pins = [(TE.test_worked_example, ()), (TE.test_gamma_zero_literal_reading_with_zero_entropy, ()),
+            (TE.test_brute_force_subsets, (0.1,))]
+    assert any(_fails(fn, *args) for fn, args in pins)
+
+
+def test_eb_descending_sort_is_caught(monkeypatch):
+    real = so.eb_select
+
+    def desc(entropy_bk, token_bk, masked_bk, block_tokens_bk, gamma):
+        return real(-np.where(np.isfinite(entropy_bk), entropy_bk, -np.inf), token_bk,
+                    masked_bk, block_tokens_bk, gamma)
+
+    monkeypatch.setattr(oracle, "eb_select", desc)
+    pins = [(TE.test_worked_example, ()), (TE.test_ties_ordered_by_position, ())]
+    assert any(_fails(fn, *args) for fn, args in pins)
