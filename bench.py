@@ -1,0 +1,512 @@
+"""Benchmark of the SBD block step on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+block attention (Eq. 5) -> LM head with fused entropy and Gumbel-max
+sampling (Eqs. 6-7) -> EB select (Eq. 3), through the C ABI of libsbd.
+The block state (masked flags, block tokens) is restored before every step
+so that every step does the same work.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...   # the fp64 oracle on host cores
+
+Prints one JSON line (rank 0).  Under torchrun every rank runs an
+independent replica on its own GPU (the block step does not shard: no data
+path collective); the time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import gen  # noqa: E402
+
+METRIC = "us per SBD block step (attention + LM head/entropy/Gumbel + EB select)"
+UNIT = "us"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ------------------------------------------------------------------ helpers
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS, "bf16_tflops": 1900.0,
+            "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+        self.marks = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), line.strip()))
+
+    def mark(self, name):
+        self.marks.append((name, time.time()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=2)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        return self.summary()
+
+    def summary(self):
+        marks = dict(self.marks)
+        t0 = marks.get("timed_start", 0.0)
+        t1 = marks.get("timed_end", time.time())
+        parsed = []
+        for t, line in self.rows:
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 10:
+                continue
+            try:
+                parsed.append(dict(t=t, sm=float(p[1]), smax=float(p[2]), util=float(p[4]),
+                                   hw=p[6], hwt=p[7], swt=p[8], pcap=p[9]))
+            except ValueError:
+                continue
+        window = "timed"
+        sel = [r for r in parsed if t0 - 0.1 <= r["t"] <= t1 + 0.1]
+        if not sel:
+            window = "bench process (timed region shorter than the 100 ms sampling period)"
+            sel = [r for r in parsed if r["util"] > 0] or parsed
+        if not sel:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        reasons = set()
+        for r in sel:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        loaded = [r["sm"] for r in sel if r["util"] > 0] or [r["sm"] for r in sel]
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(r["smax"] for r in sel),
+                "reasons": sorted(reasons), "samples": len(sel), "window": window}
+
+
+def source_sha(path: str) -> str:
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(workload: str, kernel_file: str):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, only while the kernel source is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        table = json.load(f)
+    ent = table.get(workload)
+    if not ent:
+        return None
+    if ent.get("source_sha") != source_sha(kernel_file):
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ inputs
+
+def host_inputs(w: gen.Workload, seed: int):
+    d = gen.step_inputs(w, seed, step=0, poison_tail=True)
+    return d
+
+
+def algorithmic_bytes(w: gen.Workload, d) -> dict:
+    """Bytes the method must move per step: the KV cache rows in use, block
+    K/V, Q and O once; W, the masked hidden rows, their Gumbel rows and the
+    outputs once; the EB state.  Logits are never written."""
+    e = 2 if w.dtype == "bf16" else 4
+    B, k, Hq, Hkv, D = w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim
+    L = int(np.sum(d["cache_len"]))
+    R = int(d["masked"].sum())
+    attn = (2 * L * Hkv * D + 2 * B * k * Hkv * D + 2 * B * k * Hq * D) * e + B * 4
+    head = (w.vocab * w.hidden + R * w.hidden) * e + R * w.vocab * 4 + B * k * (1 + 8)
+    eb = B * k * (4 + 4 + 1 + 4 + 1 + 4) + B * 4
+    return {"attention": attn * w.n_layers, "head": head, "eb": eb, "R": R}
+
+
+# ------------------------------------------------------------------ our arm
+
+def run_ours(args):
+    import torch
+
+    import paper_2509_04185_gb300 as sbd
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = gen.get_workload(args.workload)
+    d = host_inputs(w, args.seed)
+    dt = w.dtype
+
+    def to_dev(x):
+        x = np.ascontiguousarray(x)
+        if dt == "bf16" and x.dtype == np.uint16:
+            return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(x).to(dev)
+
+    T = {k: to_dev(d[k]) for k in ("q", "k_cache", "v_cache", "k_blk", "v_blk", "hidden", "w")}
+    T["cache_len"] = torch.from_numpy(d["cache_len"]).to(dev)
+    T["gumbel"] = torch.from_numpy(d["gumbel"]).to(dev)
+    masked0 = torch.from_numpy(d["masked"]).to(dev)
+    bt0 = torch.from_numpy(d["block_tokens"]).to(dev)
+    masked = masked0.clone()
+    bt = bt0.clone()
+    out = torch.empty_like(T["q"])
+    ent = torch.empty(masked.shape, dtype=torch.float32, device=dev)
+    tok = torch.empty(masked.shape, dtype=torch.int32, device=dev)
+    n_un = torch.empty(w.batch, dtype=torch.int32, device=dev)
+    import ctypes
+    ad = sbd.attn_desc(T["q"], T["k_cache"])
+    hd = sbd.head_desc(T["hidden"], T["w"])
+    ws_a = torch.empty(max(1, sbd.lib.sbd_block_attention_workspace_size(ctypes.byref(ad))),
+                       dtype=torch.uint8, device=dev)
+    ws_h = torch.empty(max(1, sbd.lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(hd))),
+                       dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    gamma, tau = args.gamma, args.tau
+
+    def step(ev=None):
+        masked.copy_(masked0, non_blocking=True)
+        bt.copy_(bt0, non_blocking=True)
+        if ev is not None:
+            ev[0].record(stream)
+        sbd.sbd_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"], T["k_blk"],
+                                T["v_blk"], out, workspace=ws_a, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        sbd.sbd_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau, ent, tok,
+                                    workspace=ws_h, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+        sbd.sbd_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
+        if ev is not None:
+            ev[3].record(stream)
+
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    if sbd.sbd_device_error() != 0:
+        raise RuntimeError("device error word set during warm-up")
+
+    # ---- timed region: K steps, events on the launching stream
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    if sampler:
+        sampler.mark("timed_start")
+    start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    if sampler:
+        sampler.mark("timed_end")
+    total_ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.barrier()
+        total_ms = float(t.item())
+    attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    n_accepted = int(n_un.sum().item())
+    if sbd.sbd_device_error() != 0:
+        raise RuntimeError("device error word set during the timed region")
+
+    # ---- end to end through host buffers (pinned), copies inside the region
+    e2e = None
+    if not args.skip_e2e:
+        host = {}
+        for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
+            host[k] = torch.empty_like(T[k], device="cpu").pin_memory()
+            host[k].copy_(T[k])
+        host["masked"] = masked0.cpu().pin_memory()
+        host["block_tokens"] = bt0.cpu().pin_memory()
+        res = {k: torch.empty_like(v, device="cpu").pin_memory()
+               for k, v in (("out", out), ("ent", ent), ("tok", tok), ("masked", masked),
+                            ("bt", bt), ("n_un", n_un))}
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = sum(v.numel() * v.element_size() for v in res.values())
+        n_e2e = max(1, min(args.steps, 200))
+
+        def e2e_step():
+            for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
+                T[k].copy_(host[k], non_blocking=True)
+            masked.copy_(host["masked"], non_blocking=True)
+            bt.copy_(host["block_tokens"], non_blocking=True)
+            sbd.sbd_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"],
+                                    T["k_blk"], T["v_blk"], out, workspace=ws_a, stream=stream)
+            sbd.sbd_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau, ent, tok,
+                                        workspace=ws_h, stream=stream)
+            sbd.sbd_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
+            res["out"].copy_(out, non_blocking=True)
+            res["ent"].copy_(ent, non_blocking=True)
+            res["tok"].copy_(tok, non_blocking=True)
+            res["masked"].copy_(masked, non_blocking=True)
+            res["bt"].copy_(bt, non_blocking=True)
+            res["n_un"].copy_(n_un, non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        s2 = torch.cuda.Event(enable_timing=True)
+        e2 = torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        e2.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = s2.elapsed_time(e2) / n_e2e
+        e2e = {"value": round(e2e_ms * 1000.0 / world, 3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "steps": n_e2e}
+
+    clocks = sampler.stop() if sampler else None
+
+    if rank != 0:
+        return
+    ab = algorithmic_bytes(w, d)
+    peaks, peak_src = measured_peaks()
+    head_bytes = ab["head"]
+    achieved = head_bytes / (head_ms * 1e-3) / 1e9
+    kernel_file = os.path.join(ROOT, "paper_2509_04185_gb300", "csrc", "lm_head.cu")
+    traffic = profiled_traffic(args.workload, kernel_file)
+    attn_gbs = ab["attention"] / (attn_ms * 1e-3) / 1e9
+    step_bytes = ab["attention"] + ab["head"] + ab["eb"]
+    ms_per_step = total_ms / args.steps
+    value_us = ms_per_step * 1000.0 / world
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        cpu = cpu_baseline(w, d, args)
+
+    line = {
+        "metric": METRIC,
+        "value": round(value_us, 3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 6),
+        "higher_is_better": False,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16" if dt == "bf16" else "f32",
+        "data": "synthetic (seeded generator, shapes of the workload; random-init LM head)",
+        "config": {
+            "workload": args.workload, "batch": w.batch, "block_k": w.block_k,
+            "n_q_heads": w.n_q_heads, "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+            "cache_len": w.cache_len if not isinstance(w.cache_len, tuple) else list(w.cache_len),
+            "hidden": w.hidden, "vocab": w.vocab, "masked_rows": ab["R"], "gamma": gamma,
+            "tau": tau, "parallelism": f"replicas{world}",
+            "l2": "inputs larger than L2: the 1.05 GB+ LM-head weight is streamed every step",
+        },
+        "gpu_launches": int(args.steps * launches_per_step(sbd, T, ws_a)),
+        "per_call_us": {"attention": round(attn_ms * 1000, 3), "head": round(head_ms * 1000, 3),
+                        "eb_select": round(eb_ms * 1000, 3)},
+        "step_hbm_gbs": round(step_bytes / (ms_per_step * 1e-3) / 1e9, 1),
+        "attention_hbm_gbs": round(attn_gbs, 1),
+        "tokens_committed_per_s": round(n_accepted / (ms_per_step * 1e-3) * world, 1),
+        "roofline": {
+            "kernel": "LM head call (compact_rows + head_tc_kernel tcgen05 + head_combine)",
+            "bound": "hbm", "achieved": round(achieved, 1),
+            "peak": peaks["hbm_gbs"], "peak_source": peak_src, "unit": "GB/s",
+            "frac": round(achieved / peaks["hbm_gbs"], 4),
+            "traffic": traffic, "algorithmic_bytes": int(head_bytes),
+        },
+        "clocks": clocks,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def launches_per_step(sbd, T, ws_a) -> int:
+    """Kernels of libsbd per step: attention (+ split combine), compaction,
+    LM head, head combine, EB select."""
+    import ctypes
+    ad = sbd.attn_desc(T["q"], T["k_cache"])
+    split = sbd.lib.sbd_block_attention_workspace_size(ctypes.byref(ad)) > 0
+    return (2 if split else 1) + 3 + 1
+
+
+# ------------------------------------------------------------------ oracle
+
+def _oracle_step(w, d, hkv_heads, vocab_rows, gamma, tau):
+    """The oracle on a sample of one step: attention for the query heads of
+    `hkv_heads` KV heads, the LM head over the first `vocab_rows` vocabulary
+    rows of every masked position, then the EB select of the batch."""
+    import oracle
+    dt = w.dtype
+    G = w.n_q_heads // w.n_kv_heads
+    q = oracle.widen(d["q"][:, :, : hkv_heads * G], dt)
+    kc = oracle.widen(d["k_cache"][:, :, :hkv_heads], dt)
+    vc = oracle.widen(d["v_cache"][:, :, :hkv_heads], dt)
+    kb = oracle.widen(d["k_blk"][:, :, :hkv_heads], dt)
+    vb = oracle.widen(d["v_blk"][:, :, :hkv_heads], dt)
+    oracle.block_attention(q, kc, vc, d["cache_len"], kb, vb)
+    ent, tok, _ = oracle.head_entropy_sample(oracle.widen(d["hidden"], dt), d["w"][:vocab_rows],
+                                             dt, d["masked"], d["gumbel"][:, :, :vocab_rows], tau)
+    oracle.eb_select(ent, tok, d["masked"], d["block_tokens"], gamma)
+
+
+def cpu_baseline(w, d, args, target_s: float = 15.0):
+    """Times the oracle (as it stands) on the host cores on a bounded sample
+    of the step, scaled to a full step: a fraction 1/f of the KV heads and
+    of the vocabulary.  f is the smallest power of two whose sample runs in
+    about target_s seconds (measured by a small calibration sample)."""
+    f = w.n_kv_heads
+    while f > 1 and w.vocab // f < 512:
+        f //= 2
+    t0 = time.perf_counter()
+    _oracle_step(w, d, max(1, w.n_kv_heads // f), w.vocab // f, args.gamma, args.tau)
+    t_cal = time.perf_counter() - t0
+    frac = 1.0 / f
+    while frac < 1.0 and t_cal * 2 < target_s:
+        frac *= 2
+        t_cal *= 2
+    hkv = max(1, int(round(w.n_kv_heads * frac)))
+    vrows = max(1, int(round(w.vocab * frac)))
+    t0 = time.perf_counter()
+    _oracle_step(w, d, hkv, vrows, args.gamma, args.tau)
+    dt = time.perf_counter() - t0
+    scale = 0.5 * (w.n_kv_heads / hkv) + 0.5 * (w.vocab / vrows)
+    return {"value": round(dt * scale * 1e6, 1), "unit": UNIT, "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": (f"fp64 numpy oracle on {hkv}/{w.n_kv_heads} KV heads and {vrows}/{w.vocab} "
+                       f"vocab rows of one {w.name} step ({dt:.2f} s), scaled to a full step; "
+                       f"BLAS threads = all host cores")}
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    w = gen.get_workload(args.workload)
+    d = host_inputs(w, args.seed)
+    # per-step sample sized so that warmup + steps end within about 2 minutes
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    f = w.n_kv_heads
+    while f > 1 and w.vocab // f < 512:
+        f //= 2
+    hkv = max(1, w.n_kv_heads // f)
+    vrows = w.vocab // f
+    t0 = time.perf_counter()
+    _oracle_step(w, d, hkv, vrows, args.gamma, args.tau)
+    t_cal = time.perf_counter() - t0
+    frac = 1.0 / f
+    while frac < 1.0 and t_cal * 2 < budget:
+        frac *= 2
+        t_cal *= 2
+    hkv = max(1, int(round(w.n_kv_heads * frac)))
+    vrows = max(1, int(round(w.vocab * frac)))
+    for _ in range(args.warmup):
+        _oracle_step(w, d, hkv, vrows, args.gamma, args.tau)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        _oracle_step(w, d, hkv, vrows, args.gamma, args.tau)
+        times.append(time.perf_counter() - t0)
+    scale = 0.5 * (w.n_kv_heads / hkv) + 0.5 * (w.vocab / vrows)
+    step_s = statistics.mean(times) * scale
+    value = round(step_s * 1e6, 1)
+    sample = (f"fp64 numpy oracle on {hkv}/{w.n_kv_heads} KV heads and {vrows}/{w.vocab} vocab rows "
+              f"of one {w.name} step per timed step, scaled to a full step")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic (seeded generator)",
+        "config": {"workload": args.workload, "batch": w.batch, "block_k": w.block_k,
+                   "vocab": w.vocab, "hidden": w.hidden, "gamma": args.gamma, "tau": args.tau},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llama8b_k16",
+                    choices=["llama8b_k16", "ragged_b32_k8", "qwen8b_long_k16", "tiny_f32"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--gamma", type=float, default=0.1)
+    ap.add_argument("--tau", type=float, default=1.0)
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-cpu", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -283,8 +283,10 @@ def attention_inputs(w: Workload, seed: int, layer: int = 0, poison_tail: bool =
 
 
 def lm_head_weight(w: Workload, seed: int) -> np.ndarray:
-    """W [V, H] (nn.Linear layout), N(0, w_std^2)."""
-    return store(normal_f32((w.vocab, w.hidden), seed, w.name, "w", std=w.w_std), w.dtype)
+    """W [V, H] (nn.Linear layout), N(0, w_std^2).  Keyed by shape, so the
+    workloads that share a model shape share the weight."""
+    return store(normal_f32((w.vocab, w.hidden), seed, "lm_head", w.vocab, w.hidden, "w",
+                            std=w.w_std), w.dtype)
 
 
 def hidden_states(w: Workload, seed: int, step: int = 0) -> np.ndarray:

@@ -1,0 +1,170 @@
+/*
+ * sbd.h -- C ABI of the Set Block Decoding (SBD) block step on GB300 (sm_103a).
+ *
+ * One SBD forward over a block of k positions (arXiv 2509.04185, Sec. 2.3,
+ * Eq. 5 and Algorithm 3) is served by three calls, issued in this order on
+ * one CUDA stream:
+ *
+ *   sbd_block_attention      block queries attend to the exact KV cache and,
+ *                            bidirectionally, to each other (Eq. 5; Fig. 3);
+ *   sbd_head_entropy_sample  LM head over the masked positions, reduced in
+ *                            the same kernel to a softmax entropy and a
+ *                            Gumbel-max token per position (Eqs. 6-7);
+ *   sbd_eb_select            entropy-bounded unmasking (Eq. 3).
+ *
+ * Conventions shared by every call
+ *   - Every tensor argument is a caller-owned DEVICE pointer to contiguous
+ *     row-major memory, aligned to 16 bytes.  Shapes are given in the call's
+ *     descriptor; the library never keeps a pointer after the call returns.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
+ *     enqueued asynchronously; the calls never synchronise the device.
+ *   - The library allocates no device memory.  Calls that need scratch take
+ *     a caller-owned `workspace` of at least the size returned by the
+ *     matching *_workspace_size() query; the scratch content between calls
+ *     is irrelevant (nothing needs zeroing).
+ *   - Argument errors are detected on the host before anything is enqueued
+ *     and returned as a status; sbd_last_error() then gives a one-line
+ *     explanation (per calling thread).  Launch failures return
+ *     SBD_ERR_CUDA.  No C++ exception crosses this interface.
+ *   - Device-side faults that the host cannot see before launch (a cache
+ *     length outside [0, max_cache_len], a wait that timed out) are recorded
+ *     in a device error word read by sbd_device_error().
+ *   - Calls are thread-safe; concurrent calls may share nothing but
+ *     read-only inputs (each needs its own outputs and workspace).
+ */
+#ifndef SBD_H
+#define SBD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SBD_OK = 0,
+  SBD_ERR_INVALID_ARG = 1, /* null pointer, bad size, misalignment, bad gamma/tau */
+  SBD_ERR_UNSUPPORTED = 2, /* valid but outside what the kernels implement */
+  SBD_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required */
+  SBD_ERR_CUDA = 4         /* a CUDA runtime/driver call or a launch failed */
+} sbd_status;
+
+typedef enum { SBD_DTYPE_F32 = 0, SBD_DTYPE_BF16 = 1 } sbd_dtype;
+
+/* ------------------------------------------------------------------------
+ * Block attention (Eq. 5 with the inference mask of Fig. 3 and of the
+ * FlexAttention appendix listing): every block query row i of sequence b
+ * sees the cached keys 0 .. cache_len[b]-1 and all k block keys.
+ *
+ *   q        [B, k, Hq, D]          block queries (already position-encoded)
+ *   k_cache  [B, Lmax, Hkv, D]      exact KV cache of x_<t; slots at or past
+ *   v_cache  [B, Lmax, Hkv, D]      cache_len[b] are never used (may hold NaN)
+ *   cache_len[B] int32 (device)     0 <= cache_len[b] <= Lmax
+ *   k_blk    [B, k, Hkv, D]         keys/values of the k block positions
+ *   v_blk    [B, k, Hkv, D]         (recomputed every forward, not cached)
+ *   out      [B, k, Hq, D]          attention output, same dtype as q
+ *
+ * Query head h reads KV head h / (Hq / Hkv).  s = scale * q.k with
+ * scale = desc->scale, or 1/sqrt(D) when desc->scale == 0.  All inputs share
+ * desc->dtype; accumulation is fp32.
+ * Supported: 1 <= k <= 32, D in {64, 128}, Hq % Hkv == 0,
+ * (Hq/Hkv) * k <= 128.  desc->num_splits = 0 picks the KV split count.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int32_t batch;          /* B   */
+  int32_t block_k;        /* k   */
+  int32_t n_q_heads;      /* Hq  */
+  int32_t n_kv_heads;     /* Hkv */
+  int32_t head_dim;       /* D   */
+  int32_t max_cache_len;  /* Lmax (row count of k_cache / v_cache) */
+  int32_t dtype;          /* sbd_dtype */
+  float scale;            /* 0 -> 1/sqrt(D) */
+  int32_t num_splits;     /* 0 -> automatic; else KV splits per (b, kv head) */
+} sbd_attn_desc;
+
+size_t sbd_block_attention_workspace_size(const sbd_attn_desc* desc);
+
+sbd_status sbd_block_attention(const sbd_attn_desc* desc, const void* q,
+                               const void* k_cache, const void* v_cache,
+                               const int32_t* cache_len, const void* k_blk,
+                               const void* v_blk, void* out, void* workspace,
+                               size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * LM head + entropy + Gumbel-max sample (Eqs. 6-7; Algorithm 3 "compute
+ * probabilities"), over the MASKED block positions only.  For masked
+ * position (b, i) with hidden row h = hidden[b, i, :]:
+ *   z_v      = sum_c h_c * w[v, c]                (fp32 accumulate)
+ *   entropy  = -sum_v p_v log p_v, p = softmax(z)  (nats)
+ *   token    = argmax_v (z_v + tau * gumbel[b, i, v]), lowest v on ties
+ * Logits are never written to memory.  Unmasked positions get
+ * entropy = +inf and token = -1.
+ *
+ *   hidden [B, k, H], w [V, H] (nn.Linear layout), same dtype
+ *   masked [B, k] uint8 (nonzero = masked)
+ *   gumbel [B, k, V] fp32, indexed by block position; may be NULL iff
+ *          tau == 0 (greedy); rows of unmasked positions are not read
+ *   entropy [B, k] fp32 out, token [B, k] int32 out
+ * Supported: B * k <= 256, H % 64 == 0 for bf16 (H % 4 == 0 for fp32),
+ * tau >= 0 and finite.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int32_t batch;    /* B */
+  int32_t block_k;  /* k */
+  int32_t hidden;   /* H */
+  int32_t vocab;    /* V */
+  int32_t dtype;    /* sbd_dtype of hidden and w */
+} sbd_head_desc;
+
+size_t sbd_head_entropy_sample_workspace_size(const sbd_head_desc* desc);
+
+sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden,
+                                   const void* w, const uint8_t* masked,
+                                   const float* gumbel, float tau, float* entropy,
+                                   int32_t* token, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Entropy-bounded select, entropy proxy (Eq. 3; Algorithm 3 "unmask").  Per
+ * sequence b: sort the masked positions by (entropy, position) ascending,
+ * i_1, i_2, ...; accept the first s >= 1 positions, s the largest value with
+ *   H_{i_1} + ... + H_{i_{s-1}} <= gamma     (fp32 prefix sums)
+ * capped at the number of masked positions; for each accepted i write
+ * block_tokens[b, i] = token[b, i] and masked[b, i] = 0, and set
+ * n_unmasked[b] = s (0 when nothing is masked).  Entropies of masked
+ * positions must be >= 0 (as produced by sbd_head_entropy_sample); a NaN
+ * sorts last.  Entropies/tokens of unmasked positions are not read.
+ *
+ *   entropy [B, k] fp32, token [B, k] int32   inputs
+ *   masked [B, k] uint8, block_tokens [B, k] int32 (-1 = mask)   in/out
+ *   n_unmasked [B] int32 out (may be NULL)
+ * Supported: 1 <= k <= 32, gamma >= 0 and finite.
+ * ---------------------------------------------------------------------- */
+sbd_status sbd_eb_select(int32_t batch, int32_t block_k, const float* entropy,
+                         const int32_t* token, float gamma, uint8_t* masked,
+                         int32_t* block_tokens, int32_t* n_unmasked, void* stream);
+
+/* Status name ("SBD_OK", ...). Never NULL. */
+const char* sbd_status_string(sbd_status status);
+
+/* Detail of the last failing call on this thread ("" if none). */
+const char* sbd_last_error(void);
+
+/* Reads and clears the device error word of the current device
+ * (synchronises the device).  *code = 0 when no kernel recorded a fault;
+ * otherwise a bit set of SBD_DEVERR_* values. */
+sbd_status sbd_device_error(int32_t* code);
+
+#define SBD_DEVERR_CACHE_LEN 1   /* a cache_len entry was outside [0, Lmax] */
+#define SBD_DEVERR_TIMEOUT 2     /* a bounded wait inside a kernel gave up  */
+#define SBD_DEVERR_ROWS 4        /* more masked rows than the head supports */
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t sbd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SBD_H */

@@ -1,0 +1,239 @@
+"""Python binding of libsbd, the GB300 (sm_103a) Set Block Decoding block step.
+
+Argument marshalling only: every computation runs in the CUDA kernels of
+libsbd.so (csrc/), reached through its C ABI (include/sbd.h) with ctypes.
+PyTorch supplies device memory and streams.  There is no CPU path: the
+functions require CUDA tensors, and importing this package raises if the
+library has not been built (``python -c "import __graft_entry__ as g;
+g.build()"``).
+
+The three calls of one SBD forward (arXiv 2509.04185, Eq. 5, Eqs. 6-7,
+Eq. 3 / Algorithm 3) keep the names of the C ABI:
+
+    sbd_block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk)
+    sbd_head_entropy_sample(hidden, w, masked, gumbel, tau)
+    sbd_eb_select(entropy, token, gamma, masked, block_tokens)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libsbd.so")
+
+SBD_OK = 0
+SBD_ERR_INVALID_ARG = 1
+SBD_ERR_UNSUPPORTED = 2
+SBD_ERR_WORKSPACE = 3
+SBD_ERR_CUDA = 4
+SBD_DTYPE_F32 = 0
+SBD_DTYPE_BF16 = 1
+SBD_DEVERR_CACHE_LEN = 1
+SBD_DEVERR_TIMEOUT = 2
+SBD_DEVERR_ROWS = 4
+
+# Every symbol include/sbd.h declares.
+EXPORTS = (
+    "sbd_block_attention_workspace_size",
+    "sbd_block_attention",
+    "sbd_head_entropy_sample_workspace_size",
+    "sbd_head_entropy_sample",
+    "sbd_eb_select",
+    "sbd_status_string",
+    "sbd_last_error",
+    "sbd_device_error",
+    "sbd_version",
+)
+
+
+class AttnDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("block_k", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("max_cache_len", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("scale", ctypes.c_float),
+                ("num_splits", ctypes.c_int32)]
+
+
+class HeadDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("block_k", ctypes.c_int32),
+                ("hidden", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("dtype", ctypes.c_int32)]
+
+
+class SbdError(RuntimeError):
+    def __init__(self, status: int, detail: str):
+        self.status = status
+        super().__init__(f"{_status_name(status)}: {detail}")
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it first (__graft_entry__.build())")
+    lib = ctypes.CDLL(path)
+    vp, sz, i32, f32 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int32, ctypes.c_float
+    lib.sbd_block_attention_workspace_size.argtypes = [ctypes.POINTER(AttnDesc)]
+    lib.sbd_block_attention_workspace_size.restype = sz
+    lib.sbd_block_attention.argtypes = [ctypes.POINTER(AttnDesc), vp, vp, vp, vp, vp, vp, vp,
+                                        vp, sz, vp]
+    lib.sbd_block_attention.restype = ctypes.c_int
+    lib.sbd_head_entropy_sample_workspace_size.argtypes = [ctypes.POINTER(HeadDesc)]
+    lib.sbd_head_entropy_sample_workspace_size.restype = sz
+    lib.sbd_head_entropy_sample.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp, f32, vp,
+                                            vp, vp, sz, vp]
+    lib.sbd_head_entropy_sample.restype = ctypes.c_int
+    lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
+    lib.sbd_eb_select.restype = ctypes.c_int
+    lib.sbd_status_string.argtypes = [ctypes.c_int]
+    lib.sbd_status_string.restype = ctypes.c_char_p
+    lib.sbd_last_error.argtypes = []
+    lib.sbd_last_error.restype = ctypes.c_char_p
+    lib.sbd_device_error.argtypes = [ctypes.POINTER(ctypes.c_int32)]
+    lib.sbd_device_error.restype = ctypes.c_int
+    lib.sbd_version.argtypes = []
+    lib.sbd_version.restype = i32
+    return lib
+
+
+lib = load_library()
+
+
+def _status_name(st: int) -> str:
+    return lib.sbd_status_string(st).decode()
+
+
+def _check(st: int) -> None:
+    if st != SBD_OK:
+        raise SbdError(st, lib.sbd_last_error().decode())
+
+
+# ------------------------------------------------------------------ helpers
+
+def _torch():
+    import torch
+    return torch
+
+
+def _dtype_code(t) -> int:
+    torch = _torch()
+    if t.dtype == torch.bfloat16:
+        return SBD_DTYPE_BF16
+    if t.dtype == torch.float32:
+        return SBD_DTYPE_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _need_cuda(**tensors):
+    for name, t in tensors.items():
+        if t is None:
+            continue
+        if not t.is_cuda:
+            raise ValueError(f"{name} must be a CUDA tensor (libsbd has no CPU path)")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+
+
+def _ptr(t) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    torch = _torch()
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def attn_desc(q, k_cache, scale: float = 0.0, num_splits: int = 0) -> AttnDesc:
+    B, k, Hq, D = q.shape
+    return AttnDesc(B, k, Hq, k_cache.shape[2], D, k_cache.shape[1], _dtype_code(q),
+                    float(scale), int(num_splits))
+
+
+def head_desc(hidden, w) -> HeadDesc:
+    B, k, H = hidden.shape
+    return HeadDesc(B, k, H, w.shape[0], _dtype_code(hidden))
+
+
+def _nbytes(t) -> int:
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def _workspace(nbytes: int, device, workspace=None):
+    torch = _torch()
+    if nbytes == 0:
+        return None
+    if workspace is not None and _nbytes(workspace) >= nbytes:
+        return workspace
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+# ------------------------------------------------------------------ API
+
+def sbd_block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, out=None, *,
+                        scale: float = 0.0, num_splits: int = 0, workspace=None, stream=None):
+    """Block attention (Eq. 5, inference mask of Fig. 3).  Shapes:
+    q [B,k,Hq,D], k_cache/v_cache [B,Lmax,Hkv,D], cache_len [B] int32,
+    k_blk/v_blk [B,k,Hkv,D]; returns out [B,k,Hq,D] (dtype of q)."""
+    torch = _torch()
+    _need_cuda(q=q, k_cache=k_cache, v_cache=v_cache, cache_len=cache_len, k_blk=k_blk,
+               v_blk=v_blk, out=out)
+    if cache_len.dtype != torch.int32:
+        raise TypeError("cache_len must be int32")
+    if out is None:
+        out = torch.empty_like(q)
+    d = attn_desc(q, k_cache, scale, num_splits)
+    ws = _workspace(lib.sbd_block_attention_workspace_size(ctypes.byref(d)), q.device, workspace)
+    _check(lib.sbd_block_attention(ctypes.byref(d), _ptr(q), _ptr(k_cache), _ptr(v_cache),
+                                   _ptr(cache_len), _ptr(k_blk), _ptr(v_blk), _ptr(out),
+                                   _ptr(ws), _nbytes(ws), _stream(stream)))
+    return out
+
+
+def sbd_head_entropy_sample(hidden, w, masked, gumbel, tau: float, entropy=None, token=None,
+                            *, workspace=None, stream=None):
+    """LM head + entropy + Gumbel-max token over masked positions (Eqs. 6-7).
+    hidden [B,k,H], w [V,H], masked [B,k] uint8, gumbel [B,k,V] fp32 or None
+    (tau == 0).  Returns (entropy [B,k] fp32, token [B,k] int32)."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, gumbel=gumbel, entropy=entropy, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    B, k, _ = hidden.shape
+    if entropy is None:
+        entropy = torch.empty((B, k), dtype=torch.float32, device=hidden.device)
+    if token is None:
+        token = torch.empty((B, k), dtype=torch.int32, device=hidden.device)
+    d = head_desc(hidden, w)
+    ws = _workspace(lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(d)), hidden.device,
+                    workspace)
+    _check(lib.sbd_head_entropy_sample(ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked),
+                                       _ptr(gumbel), float(tau), _ptr(entropy), _ptr(token),
+                                       _ptr(ws), _nbytes(ws), _stream(stream)))
+    return entropy, token
+
+
+def sbd_eb_select(entropy, token, gamma: float, masked, block_tokens, n_unmasked=None, *,
+                  stream=None):
+    """EB select (Eq. 3): updates masked [B,k] uint8 and block_tokens [B,k]
+    int32 in place; returns n_unmasked [B] int32."""
+    torch = _torch()
+    _need_cuda(entropy=entropy, token=token, masked=masked, block_tokens=block_tokens,
+               n_unmasked=n_unmasked)
+    B, k = masked.shape
+    if n_unmasked is None:
+        n_unmasked = torch.empty(B, dtype=torch.int32, device=masked.device)
+    _check(lib.sbd_eb_select(B, k, _ptr(entropy), _ptr(token), float(gamma), _ptr(masked),
+                             _ptr(block_tokens), _ptr(n_unmasked), _stream(stream)))
+    return n_unmasked
+
+
+def sbd_device_error() -> int:
+    """Reads and clears the device error word (synchronises the device)."""
+    code = ctypes.c_int32(0)
+    _check(lib.sbd_device_error(ctypes.byref(code)))
+    return code.value
+
+
+def sbd_version() -> int:
+    return int(lib.sbd_version())

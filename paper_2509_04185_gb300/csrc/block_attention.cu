@@ -1,0 +1,656 @@
+// Block attention of one SBD forward (arXiv 2509.04185, Eq. 5; inference
+// mask of Fig. 3): the k block queries of a sequence attend to its exact KV
+// cache (all of it lies in their past) and bidirectionally to the k block
+// keys.  Flash-decoding structure on sm_103a:
+//
+//   * one CTA per (KV split, KV head, sequence); the G = Hq/Hkv query heads
+//     that share a KV head are packed with the k block rows into one
+//     M = G*k row tile (row r = i*G + g), so each K/V byte is read once;
+//   * a producer warp streams 64-key K/V tiles into a 4-stage shared-memory
+//     ring with TMA (128-byte swizzle, completion on mbarriers); the block
+//     keys/values (not cached, k <= 32 rows) are the last tile of the last
+//     split and are copied in by the same warp;
+//   * compute warps own 16 query rows each and, when M is small, a slice of
+//     every key tile; S = Q K^T and O += P V run on bf16 mma.sync with fp32
+//     accumulators in registers; the mask (cache key < L_b, block key < k)
+//     is applied to the score registers; the online softmax keeps its row
+//     max and sum per thread and reduces them across the 4 threads of a row
+//     with shuffles;
+//   * with more than one split, each CTA writes its normalised partial
+//     output and log-sum-exp, merged by attn_combine_kernel.
+//
+// The fp32 variant (attn_f32_kernel) is a plain SIMT kernel with fp32 FMAs
+// throughout, used for fp32 inputs.
+#include <math.h>
+
+#include "sbd_internal.cuh"
+
+namespace {
+
+using namespace sbd_dev;
+
+constexpr int kTileKeys = 64;
+constexpr int kStages = 4;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------ mma helpers
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1,
+                                          uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+// D = A(16x16 bf16, row) * B(16x8 bf16, col) + D, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Address of (row, 16-byte chunk c) inside a [64 rows x 128 B] sub-tile laid
+// out by TMA with the 128-byte swizzle (chunk index XOR row % 8).
+__device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk) {
+  return base + row * 128 + (((chunk ^ (row & 7)) & 7) << 4);
+}
+
+struct AttnArgs {
+  const __nv_bfloat16* q;
+  const __nv_bfloat16* kb;
+  const __nv_bfloat16* vb;
+  const int32_t* lens;
+  __nv_bfloat16* out;        // final output (splits == 1)
+  float* part_o;             // [B, Hkv, S, M, D] (splits > 1)
+  float* part_lse;           // [B, Hkv, S, M]
+  int* err;
+  int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG;
+  float scale_log2;
+};
+
+template <int D>
+__global__ void __launch_bounds__(288, 1)
+attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                 const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
+  constexpr int kSub = D / 64;                       // 128-B column sub-tiles per row
+  constexpr int kSubBytes = kTileKeys * 128;         // 8 KB
+  constexpr int kStageBytes = 2 * kSub * kSubBytes;  // K then V
+  constexpr int kDT = D / 8;                         // n-tiles of the output
+  constexpr int kKS = D / 16;                        // k-steps of Q K^T
+
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kStages];
+  __shared__ __align__(8) uint64_t empty_bar[kStages];
+
+  const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  uint8_t* smem_gen = smem_raw + (smem_base - smem_u32(smem_raw));
+  float* merge_buf = reinterpret_cast<float*>(smem_gen + kStages * kStageBytes);
+
+  const int NW = a.MT * a.KG;                        // compute warps
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+
+  int len = a.lens[b];
+  if (len < 0 || len > a.Lmax) {
+    if (threadIdx.x == 0 && split == 0 && hkv == 0) record_error(a.err, SBD_DEVERR_CACHE_LEN);
+    len = len < 0 ? 0 : a.Lmax;
+  }
+  const int n_cache_tiles = (len + kTileKeys - 1) / kTileKeys;
+  const int n_tiles = n_cache_tiles + 1;             // + the block tile
+  const int t_begin = (int)((long long)split * n_tiles / a.splits);
+  const int t_end = (int)((long long)(split + 1) * n_tiles / a.splits);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], NW);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == NW) {
+    // ------------------------------------------------ producer warp
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap_k);
+      tma_prefetch_desc(&tmap_v);
+    }
+    int it = 0;
+    for (int t = t_begin; t < t_end; ++t, ++it) {
+      const int stage = it % kStages;
+      const uint32_t ph = (it / kStages) & 1;
+      if (!mbar_wait(&empty_bar[stage], ph ^ 1, a.err)) break;
+      const uint32_t kbase = smem_base + stage * kStageBytes;
+      const uint32_t vbase = kbase + kSub * kSubBytes;
+      if (t < n_cache_tiles) {
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
+          for (int h = 0; h < kSub; ++h) {
+            tma_load_4d(smem_gen + (kbase - smem_base) + h * kSubBytes, &tmap_k, &full_bar[stage],
+                        64 * h, hkv, t * kTileKeys, b);
+            tma_load_4d(smem_gen + (vbase - smem_base) + h * kSubBytes, &tmap_v, &full_bar[stage],
+                        64 * h, hkv, t * kTileKeys, b);
+          }
+        }
+      } else {
+        // Block keys/values: rows j < k copied, rows k..63 zero.
+        const int chunks_per_row = D / 8;                       // 16-byte chunks
+        for (int c = lane; c < kTileKeys * chunks_per_row; c += 32) {
+          const int j = c / chunks_per_row, cc = c % chunks_per_row;
+          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+          if (j < a.k) {
+            const size_t off = (((size_t)b * a.k + j) * a.Hkv + hkv) * D + cc * 8;
+            kv = *reinterpret_cast<const uint4*>(a.kb + off);
+            vv = *reinterpret_cast<const uint4*>(a.vb + off);
+          }
+          const int h = cc / 8, c8 = cc % 8;
+          const uint32_t ka = swz(kbase + h * kSubBytes, j, c8);
+          const uint32_t va = swz(vbase + h * kSubBytes, j, c8);
+          asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(ka), "r"(kv.x), "r"(kv.y),
+                       "r"(kv.z), "r"(kv.w)
+                       : "memory");
+          asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(va), "r"(vv.x), "r"(vv.y),
+                       "r"(vv.z), "r"(vv.w)
+                       : "memory");
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&full_bar[stage]);
+      }
+    }
+    // Wait for this warp's copies still in flight before the CTA may exit.
+    if (lane == 0) {
+      const int issued = it;
+      for (int q = issued - kStages > 0 ? issued - kStages : 0; q < issued; ++q)
+        mbar_wait(&full_bar[q % kStages], (q / kStages) & 1, a.err);
+    }
+  } else if (warp < NW) {
+    // ------------------------------------------------ compute warps
+    const int rt = warp % a.MT, kg = warp / a.MT;
+    const int NK = kTileKeys / a.KG;                 // keys of a tile handled by this warp
+    const int r0 = rt * 16 + (lane >> 2), r1 = r0 + 8;
+    const int qc = (lane & 3) * 2;
+
+    // Q fragments (A operand), rows r0/r1, zero for padding rows.
+    uint32_t qa[kKS][4];
+    {
+      const __nv_bfloat16* q0 = nullptr;
+      const __nv_bfloat16* q1 = nullptr;
+      if (r0 < a.M)
+        q0 = a.q + (((size_t)b * a.k + r0 / a.G) * a.Hq + hkv * a.G + r0 % a.G) * D;
+      if (r1 < a.M)
+        q1 = a.q + (((size_t)b * a.k + r1 / a.G) * a.Hq + hkv * a.G + r1 % a.G) * D;
+#pragma unroll
+      for (int ks = 0; ks < kKS; ++ks) {
+        const int c = ks * 16 + qc;
+        qa[ks][0] = q0 ? *reinterpret_cast<const uint32_t*>(q0 + c) : 0u;
+        qa[ks][1] = q1 ? *reinterpret_cast<const uint32_t*>(q1 + c) : 0u;
+        qa[ks][2] = q0 ? *reinterpret_cast<const uint32_t*>(q0 + c + 8) : 0u;
+        qa[ks][3] = q1 ? *reinterpret_cast<const uint32_t*>(q1 + c + 8) : 0u;
+      }
+    }
+
+    float o[kDT][4];
+#pragma unroll
+    for (int i = 0; i < kDT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+
+    // ldmatrix lane roles
+    const int lm = lane >> 3, lr = lane & 7;
+
+    int it = 0;
+    bool ok = true;
+    for (int t = t_begin; t < t_end; ++t, ++it) {
+      const int stage = it % kStages;
+      const uint32_t ph = (it / kStages) & 1;
+      if (!mbar_wait(&full_bar[stage], ph, a.err)) {
+        ok = false;
+        break;
+      }
+      const bool block_tile = t >= n_cache_tiles;
+      const int valid = block_tile ? a.k : min(kTileKeys, len - t * kTileKeys);
+      const uint32_t kbase = smem_base + stage * kStageBytes;
+      const uint32_t vbase = kbase + kSub * kSubBytes;
+      const int key0 = kg * NK;
+
+      // Process this warp's NK keys in chunks of 16 keys.
+      for (int kc = 0; kc < NK; kc += 16) {
+        const int j0 = key0 + kc;
+        float s[2][4];
+#pragma unroll
+        for (int n = 0; n < 2; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < kKS; ++ks) {
+          const int key = j0 + ((lm >= 2) ? 8 : 0) + lr;
+          const int d = ks * 16 + ((lm & 1) ? 8 : 0);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(swz(kbase + (d >> 6) * kSubBytes, key, (d & 63) >> 3), b0, b1, b2, b3);
+          mma_bf16(s[0], qa[ks], b0, b1);
+          mma_bf16(s[1], qa[ks], b2, b3);
+        }
+        // scale + mask in registers
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int n = 0; n < 2; ++n) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int key = j0 + n * 8 + qc + e;
+            const bool vis = key < valid;
+            s[n][e] = vis ? s[n][e] * a.scale_log2 : -INFINITY;
+            s[n][2 + e] = vis ? s[n][2 + e] * a.scale_log2 : -INFINITY;
+            mx0 = fmaxf(mx0, s[n][e]);
+            mx1 = fmaxf(mx1, s[n][2 + e]);
+          }
+        }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float mu0 = (mn0 == -INFINITY) ? 0.f : mn0;
+        const float mu1 = (mn1 == -INFINITY) ? 0.f : mn1;
+        const float al0 = exp2f(m0 - mu0), al1 = exp2f(m1 - mu1);
+        m0 = mn0;
+        m1 = mn1;
+        float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+        for (int n = 0; n < 2; ++n) {
+          s[n][0] = exp2f(s[n][0] - mu0);
+          s[n][1] = exp2f(s[n][1] - mu0);
+          s[n][2] = exp2f(s[n][2] - mu1);
+          s[n][3] = exp2f(s[n][3] - mu1);
+          ps0 += s[n][0] + s[n][1];
+          ps1 += s[n][2] + s[n][3];
+        }
+        l0 = l0 * al0 + ps0;
+        l1 = l1 * al1 + ps1;
+#pragma unroll
+        for (int i = 0; i < kDT; ++i) {
+          o[i][0] *= al0;
+          o[i][1] *= al0;
+          o[i][2] *= al1;
+          o[i][3] *= al1;
+        }
+        uint32_t pa[4];
+        pa[0] = pack_bf16(s[0][0], s[0][1]);
+        pa[1] = pack_bf16(s[0][2], s[0][3]);
+        pa[2] = pack_bf16(s[1][0], s[1][1]);
+        pa[3] = pack_bf16(s[1][2], s[1][3]);
+        // V fragments (trans), keys j0..j0+15; zero keys past `valid` so that
+        // unused cache slots (possibly NaN) never meet a zero probability.
+        const bool sanitize = j0 + 16 > valid;
+#pragma unroll
+        for (int dp = 0; dp < kDT / 2; ++dp) {
+          const int key = j0 + ((lm & 1) ? 8 : 0) + lr;
+          const int d = dp * 16 + ((lm >= 2) ? 8 : 0);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(swz(vbase + (d >> 6) * kSubBytes, key, (d & 63) >> 3), b0, b1, b2, b3);
+          if (sanitize) {
+            const int ka = j0 + qc, kb8 = j0 + 8 + qc;
+            const uint32_t m_a = (ka < valid ? 0xffffu : 0u) | (ka + 1 < valid ? 0xffff0000u : 0u);
+            const uint32_t m_b =
+                (kb8 < valid ? 0xffffu : 0u) | (kb8 + 1 < valid ? 0xffff0000u : 0u);
+            b0 &= m_a;
+            b1 &= m_b;
+            b2 &= m_a;
+            b3 &= m_b;
+          }
+          mma_bf16(o[2 * dp], pa, b0, b1);
+          mma_bf16(o[2 * dp + 1], pa, b2, b3);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[stage]);
+    }
+    (void)ok;
+
+    // Row sums across the 4 threads of a row.
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+
+    // Merge the key groups of the same row tile through shared memory.
+    if (a.KG > 1) {
+      // layout per warp: [16 rows][D] o, then [16] m, [16] l
+      float* mine = merge_buf + warp * (16 * D + 32);
+      if (kg > 0) {
+#pragma unroll
+        for (int i = 0; i < kDT; ++i) {
+          const int c = i * 8 + qc;
+          mine[(lane >> 2) * D + c] = o[i][0];
+          mine[(lane >> 2) * D + c + 1] = o[i][1];
+          mine[((lane >> 2) + 8) * D + c] = o[i][2];
+          mine[((lane >> 2) + 8) * D + c + 1] = o[i][3];
+        }
+        if ((lane & 3) == 0) {
+          mine[16 * D + (lane >> 2)] = m0;
+          mine[16 * D + (lane >> 2) + 8] = m1;
+          mine[16 * D + 16 + (lane >> 2)] = l0;
+          mine[16 * D + 16 + (lane >> 2) + 8] = l1;
+        }
+      }
+      asm volatile("bar.sync 1, %0;" ::"r"(NW * 32) : "memory");
+      if (kg == 0) {
+        for (int g2 = 1; g2 < a.KG; ++g2) {
+          const float* other = merge_buf + (g2 * a.MT + rt) * (16 * D + 32);
+          const float om0 = other[16 * D + (lane >> 2)];
+          const float om1 = other[16 * D + (lane >> 2) + 8];
+          const float ol0 = other[16 * D + 16 + (lane >> 2)];
+          const float ol1 = other[16 * D + 16 + (lane >> 2) + 8];
+          const float nm0 = fmaxf(m0, om0), nm1 = fmaxf(m1, om1);
+          const float u0 = (nm0 == -INFINITY) ? 0.f : nm0;
+          const float u1 = (nm1 == -INFINITY) ? 0.f : nm1;
+          const float sa0 = exp2f(m0 - u0), sb0 = exp2f(om0 - u0);
+          const float sa1 = exp2f(m1 - u1), sb1 = exp2f(om1 - u1);
+#pragma unroll
+          for (int i = 0; i < kDT; ++i) {
+            const int c = i * 8 + qc;
+            o[i][0] = o[i][0] * sa0 + other[(lane >> 2) * D + c] * sb0;
+            o[i][1] = o[i][1] * sa0 + other[(lane >> 2) * D + c + 1] * sb0;
+            o[i][2] = o[i][2] * sa1 + other[((lane >> 2) + 8) * D + c] * sb1;
+            o[i][3] = o[i][3] * sa1 + other[((lane >> 2) + 8) * D + c + 1] * sb1;
+          }
+          l0 = l0 * sa0 + ol0 * sb0;
+          l1 = l1 * sa1 + ol1 * sb1;
+          m0 = nm0;
+          m1 = nm1;
+        }
+      }
+    }
+
+    if (kg == 0) {
+      const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f;
+      const float inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
+      if (a.splits == 1) {
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+          const int r = rr ? r1 : r0;
+          if (r >= a.M) continue;
+          const float inv = rr ? inv1 : inv0;
+          __nv_bfloat16* dst =
+              a.out + (((size_t)b * a.k + r / a.G) * a.Hq + hkv * a.G + r % a.G) * D;
+#pragma unroll
+          for (int i = 0; i < kDT; ++i) {
+            const int c = i * 8 + qc;
+            *reinterpret_cast<uint32_t*>(dst + c) =
+                pack_bf16(o[i][2 * rr] * inv, o[i][2 * rr + 1] * inv);
+          }
+        }
+      } else {
+        const size_t pbase = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M;
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+          const int r = rr ? r1 : r0;
+          if (r >= a.M) continue;
+          const float inv = rr ? inv1 : inv0;
+          const float l = rr ? l1 : l0, m = rr ? m1 : m0;
+          float* dst = a.part_o + (pbase + r) * D;
+#pragma unroll
+          for (int i = 0; i < kDT; ++i) {
+            const int c = i * 8 + qc;
+            *reinterpret_cast<float2*>(dst + c) =
+                make_float2(o[i][2 * rr] * inv, o[i][2 * rr + 1] * inv);
+          }
+          if ((lane & 3) == 0) a.part_lse[pbase + r] = l > 0.f ? m + log2f(l) : -INFINITY;
+        }
+      }
+    }
+  }
+}
+
+// Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.
+template <typename OutT>
+__global__ void __launch_bounds__(256)
+attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
+                    OutT* __restrict__ out, int B, int k, int Hq, int Hkv, int G, int M, int D,
+                    int splits) {
+  extern __shared__ float wsm[];                     // [splits][M] weights, then [M] 1/sum
+  const int pair = blockIdx.x;                       // b * Hkv + hkv
+  const int b = pair / Hkv, hkv = pair % Hkv;
+  const float* lse = part_lse + (size_t)pair * splits * M;
+  const float* po = part_o + (size_t)pair * splits * M * D;
+  for (int r = threadIdx.x; r < M; r += blockDim.x) {
+    float mx = -INFINITY;
+    for (int s = 0; s < splits; ++s) mx = fmaxf(mx, lse[s * M + r]);
+    float sum = 0.f;
+    for (int s = 0; s < splits; ++s) {
+      const float w = (mx == -INFINITY) ? 0.f : exp2f(lse[s * M + r] - mx);
+      wsm[s * M + r] = w;
+      sum += w;
+    }
+    wsm[splits * M + r] = sum > 0.f ? 1.f / sum : 0.f;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < M * D; e += blockDim.x) {
+    const int r = e / D, d = e % D;
+    float acc = 0.f;
+    for (int s = 0; s < splits; ++s) acc += wsm[s * M + r] * po[((size_t)s * M + r) * D + d];
+    acc *= wsm[splits * M + r];
+    const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + d;
+    if constexpr (sizeof(OutT) == 2)
+      out[o] = __float2bfloat16_rn(acc);
+    else
+      out[o] = acc;
+  }
+}
+
+// ------------------------------------------------------------ fp32 variant
+// One CTA per (query row i, query head, sequence); keys in chunks of 128
+// with an online softmax; every product and sum in fp32 FMAs.
+__global__ void __launch_bounds__(128)
+attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
+                const float* __restrict__ vc, const int32_t* __restrict__ lens,
+                const float* __restrict__ kb, const float* __restrict__ vb,
+                float* __restrict__ out, int* err, int k, int Hq, int Hkv, int D, int Lmax,
+                float scale_log2, int splits, float* part_o, float* part_lse) {
+  __shared__ float qs[128];
+  __shared__ float ps[128];
+  __shared__ float red[4];
+  const int i = blockIdx.x, hq = blockIdx.y, b = blockIdx.z;
+  const int G = Hq / Hkv, hkv = hq / G;
+  const int tid = threadIdx.x;
+  int len = lens[b];
+  if (len < 0 || len > Lmax) {
+    if (tid == 0) sbd_dev::record_error(err, SBD_DEVERR_CACHE_LEN);
+    len = len < 0 ? 0 : Lmax;
+  }
+  const float* qrow = q + (((size_t)b * k + i) * Hq + hq) * D;
+  if (tid < D) qs[tid] = qrow[tid];
+  __syncthreads();
+  const int total = len + k;
+  float m = -INFINITY, l = 0.f, acc = 0.f;   // acc: output element d = tid
+  for (int c0 = 0; c0 < total; c0 += 128) {
+    const int u = c0 + tid;
+    float s = -INFINITY;
+    if (u < total) {
+      const float* key = (u < len) ? kc + (((size_t)b * Lmax + u) * Hkv + hkv) * D
+                                   : kb + (((size_t)b * k + (u - len)) * Hkv + hkv) * D;
+      float dot = 0.f;
+      for (int d = 0; d < D; ++d) dot = fmaf(qs[d], key[d], dot);
+      s = dot * scale_log2;
+    }
+    // block max
+    float mx = sbd_dev::warp_max(s);
+    if ((tid & 31) == 0) red[tid >> 5] = mx;
+    __syncthreads();
+    mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    __syncthreads();
+    const float mn = fmaxf(m, mx);
+    const float alpha = (m == -INFINITY) ? 0.f : exp2f(m - mn);
+    const float p = (s == -INFINITY) ? 0.f : exp2f(s - mn);
+    ps[tid] = p;
+    float psum = sbd_dev::warp_sum(p);
+    if ((tid & 31) == 0) red[tid >> 5] = psum;
+    __syncthreads();
+    psum = (red[0] + red[1]) + (red[2] + red[3]);
+    l = l * alpha + psum;
+    m = mn;
+    if (tid < D) {
+      acc *= alpha;
+      const int n = min(128, total - c0);
+      for (int j = 0; j < n; ++j) {
+        const int uu = c0 + j;
+        const float* val = (uu < len) ? vc + (((size_t)b * Lmax + uu) * Hkv + hkv) * D
+                                      : vb + (((size_t)b * k + (uu - len)) * Hkv + hkv) * D;
+        acc = fmaf(ps[j], val[tid], acc);
+      }
+    }
+    __syncthreads();
+  }
+  if (tid < D) out[(((size_t)b * k + i) * Hq + hq) * D + tid] = acc / l;
+  (void)splits;
+  (void)part_o;
+  (void)part_lse;
+}
+
+}  // namespace
+
+namespace sbd {
+
+static int choose_splits(int pairs, int n_tiles_max, int sms) {
+  if (pairs >= 2 * sms) return 1;
+  int max_s = n_tiles_max / 2;
+  if (max_s < 1) max_s = 1;
+  if (max_s > 32) max_s = 32;
+  int best = 1;
+  double best_eff = 0.0;
+  for (int s = 1; s <= max_s; ++s) {
+    const long long ctas = (long long)pairs * s;
+    const long long waves = (ctas + sms - 1) / sms;
+    const double eff = (double)ctas / (double)(waves * sms);
+    if (eff > best_eff + 0.02) {
+      best_eff = eff;
+      best = s;
+    }
+  }
+  return best;
+}
+
+AttnPlan attn_plan(const sbd_attn_desc& d) {
+  AttnPlan p;
+  p.B = d.batch;
+  p.k = d.block_k;
+  p.Hq = d.n_q_heads;
+  p.Hkv = d.n_kv_heads;
+  p.G = d.n_q_heads / d.n_kv_heads;
+  p.D = d.head_dim;
+  p.Lmax = d.max_cache_len;
+  p.M = p.G * p.k;
+  p.bf16 = d.dtype == SBD_DTYPE_BF16;
+  const float scale = d.scale != 0.f ? d.scale : 1.0f / sqrtf((float)d.head_dim);
+  p.scale_log2 = scale * kLog2e;
+  if (!p.bf16) {
+    p.splits = 1;
+  } else if (d.num_splits > 0) {
+    p.splits = d.num_splits;
+  } else {
+    const int tiles = (p.Lmax + kTileKeys - 1) / kTileKeys + 1;
+    p.splits = choose_splits(p.B * p.Hkv, tiles, num_sms());
+  }
+  return p;
+}
+
+size_t attn_workspace_bytes(const AttnPlan& p) {
+  if (p.splits <= 1) return 0;
+  const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
+  return align_up(n * p.D * sizeof(float), 256) + align_up(n * sizeof(float), 256);
+}
+
+static size_t attn_smem_bytes(int D, int NW, int KG) {
+  const size_t stages = (size_t)kStages * 2 * (D / 64) * kTileKeys * 128;
+  const size_t merge = KG > 1 ? (size_t)NW * (16 * D + 32) * sizeof(float) : 0;
+  return 1024 + stages + merge;
+}
+
+sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const void* vc,
+                       const int32_t* lens, const void* kb, const void* vb, void* out, void* ws,
+                       cudaStream_t st) {
+  if (p.B == 0) return SBD_OK;
+  int* err = device_error_word();
+  if (!p.bf16) {
+    dim3 grid(p.k, p.Hq, p.B);
+    attn_f32_kernel<<<grid, 128, 0, st>>>(
+        (const float*)q, (const float*)kc, (const float*)vc, lens, (const float*)kb,
+        (const float*)vb, (float*)out, err, p.k, p.Hq, p.Hkv, p.D, p.Lmax, p.scale_log2, 1,
+        nullptr, nullptr);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? SBD_OK : cuda_fail(e, "attn_f32_kernel launch");
+  }
+
+  // 4-D tensor maps over the caches: dims (D, Hkv, Lmax, B), 64x64 boxes.
+  CUtensorMap tk, tv;
+  const uint64_t dims[4] = {(uint64_t)p.D, (uint64_t)p.Hkv, (uint64_t)p.Lmax, (uint64_t)p.B};
+  const uint64_t strides[3] = {(uint64_t)p.D * 2, (uint64_t)p.Hkv * p.D * 2,
+                               (uint64_t)p.Lmax * p.Hkv * p.D * 2};
+  const uint32_t box[4] = {64, 1, (uint32_t)kTileKeys, 1};
+  sbd_status s = encode_tensor_map(&tk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, (void*)kc, dims,
+                                   strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+  if (s != SBD_OK) return s;
+  s = encode_tensor_map(&tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, (void*)vc, dims, strides, box,
+                        CU_TENSOR_MAP_SWIZZLE_128B);
+  if (s != SBD_OK) return s;
+
+  AttnArgs a;
+  a.q = (const __nv_bfloat16*)q;
+  a.kb = (const __nv_bfloat16*)kb;
+  a.vb = (const __nv_bfloat16*)vb;
+  a.lens = lens;
+  a.out = (__nv_bfloat16*)out;
+  a.err = err;
+  a.B = p.B;
+  a.k = p.k;
+  a.Hq = p.Hq;
+  a.Hkv = p.Hkv;
+  a.G = p.G;
+  a.M = p.M;
+  a.Lmax = p.Lmax;
+  a.splits = p.splits;
+  a.MT = (p.M + 15) / 16;
+  a.KG = a.MT >= 4 ? 1 : 4 / a.MT;
+  a.scale_log2 = p.scale_log2;
+  const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
+  a.part_o = (float*)ws;
+  a.part_lse = p.splits > 1 ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
+
+  const int NW = a.MT * a.KG;
+  const size_t smem = attn_smem_bytes(p.D, NW, a.KG);
+  dim3 grid(p.splits, p.Hkv, p.B);
+  dim3 block(32 * (NW + 1));
+  cudaError_t e;
+  if (p.D == 128) {
+    e = cudaFuncSetAttribute(attn_bf16_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_bf16_kernel)");
+    attn_bf16_kernel<128><<<grid, block, smem, st>>>(tk, tv, a);
+  } else {
+    e = cudaFuncSetAttribute(attn_bf16_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_bf16_kernel)");
+    attn_bf16_kernel<64><<<grid, block, smem, st>>>(tk, tv, a);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "attn_bf16_kernel launch");
+  if (p.splits > 1) {
+    const size_t cs = ((size_t)p.splits + 1) * p.M * sizeof(float);
+    attn_combine_kernel<__nv_bfloat16><<<p.B * p.Hkv, 256, cs, st>>>(
+        a.part_o, a.part_lse, (__nv_bfloat16*)out, p.B, p.k, p.Hq, p.Hkv, p.G, p.M, p.D,
+        p.splits);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "attn_combine_kernel launch");
+  }
+  return SBD_OK;
+}
+
+}  // namespace sbd

@@ -1,0 +1,651 @@
+// LM head over the masked block positions, reduced in the same kernel to a
+// softmax entropy and a Gumbel-max token per position (arXiv 2509.04185,
+// Eqs. 6-7 and Algorithm 3 "compute probabilities"; EB input of Eq. 3).
+//
+// Kernels, in launch order on one stream:
+//   compact_rows_kernel  gathers the hidden rows of masked positions into a
+//                        dense [rows_alloc, H] buffer and a row map; writes
+//                        entropy = +inf / token = -1 for unmasked positions;
+//   head_tc_kernel       (bf16) persistent tcgen05 GEMM, swap-AB: 128 vocab
+//                        rows of W are the M side (A, K-major), the masked
+//                        hidden rows the N side (B, K-major).  A warp streams
+//                        W and hidden tiles into a shared-memory ring with
+//                        TMA; one thread issues tcgen05.mma into a
+//                        double-buffered fp32 accumulator in tensor memory;
+//                        four epilogue warps read it back with tcgen05.ld and
+//                        reduce every logit column to running statistics
+//                        (max, sum of exponentials, entropy numerator, best
+//                        Gumbel score and id) -- logits never reach HBM;
+//   head_f32_kernel      (fp32) the same reduction over exact fp32 FMAs;
+//   head_combine_kernel  merges the per-CTA statistics of each row into the
+//                        entropy (nats) and the token.
+#include <math.h>
+
+#include "sbd_internal.cuh"
+
+namespace {
+
+using namespace sbd_dev;
+
+constexpr int kBM = 128;              // vocab rows per tile (MMA M)
+constexpr int kBK = 64;               // hidden columns per stage (one 128-B swizzle atom)
+constexpr int kABytes = kBM * kBK * 2;
+constexpr int kMaxStages = 16;
+constexpr int kHeadThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// ------------------------------------------------------------ tcgen05 PTX
+__device__ __forceinline__ void tc_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrives once on the mbarrier when every tcgen05 op issued so far by this
+// thread has completed.
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+// 32 lanes x 16 consecutive 32-bit columns: thread t gets lane (base + t).
+__device__ __forceinline__ void tc_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tc_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand laid out by TMA with the
+// 128-byte swizzle, rows 128 B apart, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t smem_addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr & 0x3FFFFu) >> 4);   // start address
+  d |= (uint64_t)(16u >> 4) << 16;                 // leading byte offset (unused here)
+  d |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: 8 rows x 128 B
+  d |= (uint64_t)1u << 46;                         // descriptor version (tcgen05)
+  d |= (uint64_t)2u << 61;                         // 128-byte swizzle
+  return d;
+}
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4)                  // D format: f32
+         | (1u << 7)                // A format: bf16
+         | (1u << 10)               // B format: bf16
+         | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ------------------------------------------------------------ epilogue math
+// Reduces one logit column over the 32 lanes of a warp (lane = vocab id v).
+__device__ __forceinline__ RowStats warp_column_stats(float z, bool valid, float g, float tau,
+                                                      int v) {
+  const float y = valid ? z * kLog2e : -INFINITY;
+  const float m = warp_max(y);
+  float e = 0.f, t = 0.f;
+  if (valid && m != -INFINITY) {
+    const float dy = y - m;
+    e = exp2f(dy);
+    t = e * dy;
+  }
+  RowStats r;
+  r.m = m;
+  r.S = warp_sum(e);
+  r.T = warp_sum(t);
+  float best = valid ? fmaf(tau, g, z) : -INFINITY;
+  int idx = valid ? v : 0x7fffffff;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+    if (ob > best || (ob == best && oi < idx)) {
+      best = ob;
+      idx = oi;
+    }
+  }
+  r.best = best;
+  r.idx = idx;
+  return r;
+}
+
+struct StatsRef {
+  float4* msTb;   // (m, S, T, best)
+  int* idx;
+};
+__device__ __forceinline__ RowStats load_stats(const StatsRef& s, int i) {
+  const float4 v = s.msTb[i];
+  RowStats r;
+  r.m = v.x;
+  r.S = v.y;
+  r.T = v.z;
+  r.best = v.w;
+  r.idx = s.idx[i];
+  return r;
+}
+__device__ __forceinline__ void store_stats(const StatsRef& s, int i, const RowStats& r) {
+  s.msTb[i] = make_float4(r.m, r.S, r.T, r.best);
+  s.idx[i] = r.idx;
+}
+
+// ------------------------------------------------------------ compaction
+__global__ void __launch_bounds__(256)
+compact_rows_kernel(const uint8_t* __restrict__ hidden, const uint8_t* __restrict__ masked,
+                    int BK, int row_bytes, uint8_t* __restrict__ hidden_c,
+                    int32_t* __restrict__ row_map, int32_t* __restrict__ n_rows,
+                    float* __restrict__ entropy, int32_t* __restrict__ token) {
+  grid_dependents_launch();
+  const int row = blockIdx.x;
+  const int t = threadIdx.x;
+  const bool mt = t < BK && masked[t] != 0;
+  const int before = __syncthreads_count(mt && t < row);
+  const int total = __syncthreads_count(mt);
+  int dst;
+  bool copy = false;
+  if (row < BK) {
+    if (masked[row]) {
+      dst = before;
+      copy = true;
+      if (t == 0) row_map[dst] = row;
+    } else {
+      dst = total + (row - before);
+      if (t == 0) {
+        entropy[row] = INFINITY;
+        token[row] = -1;
+      }
+    }
+  } else {
+    dst = row;
+  }
+  const int n16 = row_bytes / 16;
+  uint4* out = reinterpret_cast<uint4*>(hidden_c + (size_t)dst * row_bytes);
+  const uint4* in = reinterpret_cast<const uint4*>(hidden + (size_t)row * row_bytes);
+  for (int c = t; c < n16; c += blockDim.x) out[c] = copy ? in[c] : make_uint4(0, 0, 0, 0);
+  if (row == 0 && t == 0) *n_rows = total;
+}
+
+// ------------------------------------------------------------ bf16 tcgen05
+struct HeadArgs {
+  const float* gumbel;
+  const int32_t* row_map;
+  const int32_t* n_rows;
+  float4* part_msTb;     // [gridDim.x][rows_alloc]
+  int32_t* part_idx;
+  int* err;
+  int V, H, rows_alloc, n_tiles, stages;
+  uint32_t tmem_cols;
+  float tau;
+};
+
+__global__ void __launch_bounds__(kHeadThreads, 1)
+head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
+               const __grid_constant__ CUtensorMap tmap_h, const HeadArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t tmem_full[2];
+  __shared__ __align__(8) uint64_t tmem_empty[2];
+  __shared__ uint32_t tmem_base_sh;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (sbase - smem_u32(smem_raw));
+  const int b_bytes = a.rows_alloc * kBK * 2;
+  const int stage_bytes = kABytes + b_bytes;
+  // epilogue scratch after the ring
+  uint8_t* ep = gbase + (size_t)a.stages * stage_bytes;
+  StatsRef wstats[4];
+  for (int w = 0; w < 4; ++w) {
+    wstats[w].msTb = reinterpret_cast<float4*>(ep) + w * a.rows_alloc;
+    wstats[w].idx = reinterpret_cast<int*>(ep + (size_t)4 * a.rows_alloc * sizeof(float4)) +
+                    w * a.rows_alloc;
+  }
+  int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * a.rows_alloc * (sizeof(float4) + 4));
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < a.stages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tmem_full[i], 1);
+      mbar_init(&tmem_empty[i], 128);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_h);
+  }
+  if (warp == 1) tc_alloc(&tmem_base_sh, a.tmem_cols);
+  // Everything below reads what the compaction kernel wrote.
+  grid_dependency_wait();
+  const int R = *a.n_rows;
+  if (warp >= 2) {
+    const int te = threadIdx.x - 64;
+    for (int i = te; i < a.rows_alloc; i += 128) {
+      rmap[i] = i < R ? a.row_map[i] : 0;
+      for (int w = 0; w < 4; ++w) store_stats(wstats[w], i, rowstats_empty());
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_base_sh;
+  const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
+  const int num_kb = a.H / kBK;
+
+  if (R > 0) {
+    if (warp == 0) {
+      // ------------------------------------------------ TMA producer
+      if (lane == 0) {
+        const uint64_t policy = l2_policy_evict_first();
+        int it = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += gridDim.x) {
+          for (int kb = 0; kb < num_kb; ++kb, ++it) {
+            const int s = it % a.stages;
+            const uint32_t ph = (it / a.stages) & 1;
+            if (!mbar_wait(&empty_bar[s], ph ^ 1, a.err)) {
+              ok = false;
+              break;
+            }
+            uint8_t* st = gbase + (size_t)s * stage_bytes;
+            mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+            tma_load_2d_hint(st, &tmap_w, &full_bar[s], kb * kBK, tile * kBM, policy);
+            tma_load_2d(st + kABytes, &tmap_h, &full_bar[s], kb * kBK, 0);
+          }
+        }
+        // copies still in flight must land before the CTA exits
+        for (int q = it - a.stages > 0 ? it - a.stages : 0; q < it; ++q)
+          mbar_wait(&full_bar[q % a.stages], (q / a.stages) & 1, a.err);
+      }
+    } else if (warp == 1) {
+      // ------------------------------------------------ MMA issuer
+      if (lane == 0) {
+        const uint32_t idesc = idesc_bf16_f32(kBM, n_eff);
+        int it = 0, local = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += gridDim.x, ++local) {
+          const int acc = local & 1;
+          const uint32_t use = (uint32_t)(local >> 1);
+          if (!mbar_wait(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + (uint32_t)(acc * a.rows_alloc);
+          for (int kb = 0; kb < num_kb; ++kb, ++it) {
+            const int s = it % a.stages;
+            const uint32_t ph = (it / a.stages) & 1;
+            if (!mbar_wait(&full_bar[s], ph, a.err)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = sbase + (uint32_t)(s * stage_bytes);
+            const uint64_t adesc = sw128_kmajor_desc(st);
+            const uint64_t bdesc = sw128_kmajor_desc(st + kABytes);
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              tc_mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
+            tc_commit(&empty_bar[s]);
+          }
+          if (ok) tc_commit(&tmem_full[acc]);
+        }
+      }
+    } else {
+      // ------------------------------------------------ epilogue warps
+      const int ew = warp - 2;                 // 0..3
+      const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
+      const bool noisy = a.tau != 0.f && a.gumbel != nullptr;
+      int local = 0;
+      for (int tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++local) {
+        const int acc = local & 1;
+        const uint32_t use = (uint32_t)(local >> 1);
+        const int v = tile * kBM + quad * 32 + lane;
+        const bool valid = v < a.V;
+        for (int c0 = 0; c0 < R; c0 += 16) {
+          float g[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            g[j] = 0.f;
+            if (noisy && valid && c0 + j < R) g[j] = __ldg(a.gumbel + (size_t)rmap[c0 + j] * a.V + v);
+          }
+          if (c0 == 0) {
+            if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
+            tc_fence_after();
+          }
+          uint32_t r[16];
+          tc_ld_32x32b_x16(tmem_base + ((uint32_t)(quad * 32) << 16) +
+                               (uint32_t)(acc * a.rows_alloc + c0),
+                           r);
+          tc_wait_ld();
+          RowStats mine = rowstats_empty();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            if (c0 + j < R) {
+              const RowStats cs = warp_column_stats(__uint_as_float(r[j]), valid, g[j], a.tau, v);
+              if (lane == j) mine = cs;
+            }
+          }
+          if (lane < 16 && c0 + lane < R) {
+            const int col = c0 + lane;
+            store_stats(wstats[ew], col, rowstats_merge(load_stats(wstats[ew], col), mine));
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&tmem_empty[acc]);
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const int te = threadIdx.x - 64;
+      for (int col = te; col < R; col += 128) {
+        RowStats s = load_stats(wstats[0], col);
+        for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats[w], col));
+        const size_t o = (size_t)blockIdx.x * a.rows_alloc + col;
+        a.part_msTb[o] = make_float4(s.m, s.S, s.T, s.best);
+        a.part_idx[o] = s.idx;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tc_dealloc(tmem_base, a.tmem_cols);
+  }
+}
+
+// ------------------------------------------------------------ fp32 SIMT
+// One CTA per 128 vocab rows; z by sequential fp32 FMAs over H; the same
+// column statistics as the tensor-core epilogue.
+__global__ void __launch_bounds__(128)
+head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
+                const float* __restrict__ gumbel, const int32_t* __restrict__ row_map,
+                const int32_t* __restrict__ n_rows, float tau, int V, int H, int rows_alloc,
+                float4* __restrict__ part_msTb, int32_t* __restrict__ part_idx) {
+  grid_dependency_wait();
+  __shared__ float4 sm[4][32];
+  __shared__ int si[4][32];
+  const int R = *n_rows;
+  const int v = blockIdx.x * 128 + threadIdx.x;
+  const bool valid = v < V;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool noisy = tau != 0.f && gumbel != nullptr;
+  const float* wrow = w + (size_t)(valid ? v : 0) * H;
+  for (int r0 = 0; r0 < R; r0 += 32) {
+    const int nr = min(32, R - r0);
+    RowStats mine = rowstats_empty();
+    for (int j = 0; j < nr; ++j) {
+      const float* h = hidden_c + (size_t)(r0 + j) * H;
+      float z = 0.f;
+      for (int c = 0; c < H; ++c) z = fmaf(h[c], wrow[c], z);
+      const float g = (noisy && valid) ? gumbel[(size_t)row_map[r0 + j] * V + v] : 0.f;
+      const RowStats cs = warp_column_stats(z, valid, g, tau, v);
+      if (lane == j) mine = cs;
+    }
+    if (lane < nr) {
+      sm[warp][lane] = make_float4(mine.m, mine.S, mine.T, mine.best);
+      si[warp][lane] = mine.idx;
+    }
+    __syncthreads();
+    if (threadIdx.x < nr) {
+      RowStats s;
+      s.m = sm[0][threadIdx.x].x;
+      s.S = sm[0][threadIdx.x].y;
+      s.T = sm[0][threadIdx.x].z;
+      s.best = sm[0][threadIdx.x].w;
+      s.idx = si[0][threadIdx.x];
+      for (int w2 = 1; w2 < 4; ++w2) {
+        RowStats o;
+        o.m = sm[w2][threadIdx.x].x;
+        o.S = sm[w2][threadIdx.x].y;
+        o.T = sm[w2][threadIdx.x].z;
+        o.best = sm[w2][threadIdx.x].w;
+        o.idx = si[w2][threadIdx.x];
+        s = rowstats_merge(s, o);
+      }
+      const size_t o = (size_t)blockIdx.x * rows_alloc + r0 + threadIdx.x;
+      part_msTb[o] = make_float4(s.m, s.S, s.T, s.best);
+      part_idx[o] = s.idx;
+    }
+    __syncthreads();
+  }
+}
+
+// ------------------------------------------------------------ combine
+// One warp per masked row: merge the per-CTA statistics, then
+// H = ln 2 * (log2 S - T / S)  (nats) and the winning token.
+__global__ void __launch_bounds__(128)
+head_combine_kernel(const float4* __restrict__ part_msTb, const int32_t* __restrict__ part_idx,
+                    int n_parts, int rows_alloc, const int32_t* __restrict__ row_map,
+                    const int32_t* __restrict__ n_rows, float* __restrict__ entropy,
+                    int32_t* __restrict__ token) {
+  grid_dependency_wait();
+  const int r = blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= *n_rows) return;
+  RowStats s = rowstats_empty();
+  for (int c = lane; c < n_parts; c += 32) {
+    const float4 v = part_msTb[(size_t)c * rows_alloc + r];
+    RowStats o;
+    o.m = v.x;
+    o.S = v.y;
+    o.T = v.z;
+    o.best = v.w;
+    o.idx = part_idx[(size_t)c * rows_alloc + r];
+    s = rowstats_merge(s, o);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    RowStats t;
+    t.m = __shfl_xor_sync(0xffffffffu, s.m, o);
+    t.S = __shfl_xor_sync(0xffffffffu, s.S, o);
+    t.T = __shfl_xor_sync(0xffffffffu, s.T, o);
+    t.best = __shfl_xor_sync(0xffffffffu, s.best, o);
+    t.idx = __shfl_xor_sync(0xffffffffu, s.idx, o);
+    s = rowstats_merge(s, t);
+  }
+  if (lane == 0) {
+    const int row = row_map[r];
+    entropy[row] = kLn2 * (log2f(s.S) - s.T / s.S);
+    token[row] = s.idx;
+  }
+}
+
+// ------------------------------------------------------------ workspace
+struct HeadWs {
+  uint8_t* hidden_c;
+  int32_t* row_map;
+  int32_t* n_rows;
+  float4* part_msTb;
+  int32_t* part_idx;
+  size_t bytes;
+};
+
+HeadWs head_ws_layout(const sbd::HeadPlan& p, void* base) {
+  HeadWs w;
+  const uintptr_t c = reinterpret_cast<uintptr_t>(base);
+  size_t off = 0;
+  const size_t elem = p.bf16 ? 2 : 4;
+  w.hidden_c = reinterpret_cast<uint8_t*>(c + off);
+  off = sbd::align_up(off + (size_t)p.rows_alloc * p.H * elem, 256);
+  w.row_map = reinterpret_cast<int32_t*>(c + off);
+  off = sbd::align_up(off + (size_t)p.rows_alloc * 4, 256);
+  w.n_rows = reinterpret_cast<int32_t*>(c + off);
+  off = sbd::align_up(off + 4, 256);
+  w.part_msTb = reinterpret_cast<float4*>(c + off);
+  off = sbd::align_up(off + (size_t)p.n_ctas * p.rows_alloc * sizeof(float4), 256);
+  w.part_idx = reinterpret_cast<int32_t*>(c + off);
+  off = sbd::align_up(off + (size_t)p.n_ctas * p.rows_alloc * 4, 256);
+  w.bytes = off;
+  return w;
+}
+
+int head_stages(int rows_alloc) {
+  const int stage_bytes = kABytes + rows_alloc * kBK * 2;
+  const int ep_bytes = 4 * rows_alloc * (16 + 4) + rows_alloc * 4;
+  const int budget = 220 * 1024 - 1024 - ep_bytes;
+  int s = budget / stage_bytes;
+  if (s > kMaxStages) s = kMaxStages;
+  return s;
+}
+
+size_t head_smem_bytes(int rows_alloc, int stages) {
+  const size_t stage_bytes = kABytes + (size_t)rows_alloc * kBK * 2;
+  return 1024 + stages * stage_bytes + (size_t)4 * rows_alloc * (16 + 4) + rows_alloc * 4;
+}
+
+}  // namespace
+
+namespace sbd {
+
+HeadPlan head_plan(const sbd_head_desc& d) {
+  HeadPlan p;
+  p.B = d.batch;
+  p.k = d.block_k;
+  p.H = d.hidden;
+  p.V = d.vocab;
+  p.bf16 = d.dtype == SBD_DTYPE_BF16;
+  const int bk = d.batch * d.block_k;
+  p.rows_alloc = bk <= 16 ? 16 : ((bk + 15) / 16) * 16;
+  const int n_tiles = (d.vocab + kBM - 1) / kBM;
+  if (p.bf16) {
+    const int sms = num_sms();
+    p.n_ctas = n_tiles < sms ? n_tiles : sms;
+  } else {
+    p.n_ctas = n_tiles;
+  }
+  return p;
+}
+
+size_t head_workspace_bytes(const HeadPlan& p) { return head_ws_layout(p, nullptr).bytes; }
+
+static sbd_status launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                             void** args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelExC(&cfg, fn, args);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernelExC");
+  return SBD_OK;
+}
+
+sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
+                       const uint8_t* masked, const float* gumbel, float tau, float* entropy,
+                       int32_t* token, void* ws, cudaStream_t st) {
+  const int BK = p.B * p.k;
+  if (BK == 0) return SBD_OK;
+  HeadWs W = head_ws_layout(p, ws);
+  const int elem = p.bf16 ? 2 : 4;
+  compact_rows_kernel<<<p.rows_alloc, 256, 0, st>>>((const uint8_t*)hidden, masked, BK,
+                                                    p.H * elem, W.hidden_c, W.row_map, W.n_rows,
+                                                    entropy, token);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "compact_rows_kernel launch");
+
+  int* err = device_error_word();
+  sbd_status s;
+  if (p.bf16) {
+    CUtensorMap tw, th;
+    {
+      const uint64_t dims[2] = {(uint64_t)p.H, (uint64_t)p.V};
+      const uint64_t strides[1] = {(uint64_t)p.H * 2};
+      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)kBM};
+      s = encode_tensor_map(&tw, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)w, dims, strides,
+                            box, CU_TENSOR_MAP_SWIZZLE_128B);
+      if (s != SBD_OK) return s;
+    }
+    {
+      const uint64_t dims[2] = {(uint64_t)p.H, (uint64_t)p.rows_alloc};
+      const uint64_t strides[1] = {(uint64_t)p.H * 2};
+      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)p.rows_alloc};
+      s = encode_tensor_map(&th, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)W.hidden_c, dims,
+                            strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+      if (s != SBD_OK) return s;
+    }
+    HeadArgs a;
+    a.gumbel = gumbel;
+    a.row_map = W.row_map;
+    a.n_rows = W.n_rows;
+    a.part_msTb = W.part_msTb;
+    a.part_idx = W.part_idx;
+    a.err = err;
+    a.V = p.V;
+    a.H = p.H;
+    a.rows_alloc = p.rows_alloc;
+    a.n_tiles = (p.V + kBM - 1) / kBM;
+    a.stages = head_stages(p.rows_alloc);
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(2 * p.rows_alloc)) cols <<= 1;
+    a.tmem_cols = cols;
+    a.tau = tau;
+    const size_t smem = head_smem_bytes(p.rows_alloc, a.stages);
+    e = cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
+    void* args[] = {(void*)&tw, (void*)&th, (void*)&a};
+    s = launch_pdl((const void*)head_tc_kernel, dim3(p.n_ctas), dim3(kHeadThreads), smem, st,
+                   args);
+    if (s != SBD_OK) return s;
+  } else {
+    const float* hc = (const float*)W.hidden_c;
+    const float* wf = (const float*)w;
+    const int32_t* rm = W.row_map;
+    const int32_t* nr = W.n_rows;
+    int V = p.V, H = p.H, ra = p.rows_alloc;
+    float4* pm = W.part_msTb;
+    int32_t* pi = W.part_idx;
+    void* args[] = {(void*)&hc, (void*)&wf, (void*)&gumbel, (void*)&rm, (void*)&nr,
+                    (void*)&tau, (void*)&V,  (void*)&H,      (void*)&ra, (void*)&pm,
+                    (void*)&pi};
+    s = launch_pdl((const void*)head_f32_kernel, dim3(p.n_ctas), dim3(128), 0, st, args);
+    if (s != SBD_OK) return s;
+  }
+  {
+    const float4* pm = W.part_msTb;
+    const int32_t* pi = W.part_idx;
+    int np = p.n_ctas, ra = p.rows_alloc;
+    const int32_t* rm = W.row_map;
+    const int32_t* nr = W.n_rows;
+    void* args[] = {(void*)&pm, (void*)&pi, (void*)&np, (void*)&ra,
+                    (void*)&rm, (void*)&nr, (void*)&entropy, (void*)&token};
+    s = launch_pdl((const void*)head_combine_kernel, dim3((p.rows_alloc + 3) / 4), dim3(128), 0,
+                   st, args);
+    if (s != SBD_OK) return s;
+  }
+  return SBD_OK;
+}
+
+}  // namespace sbd

@@ -1,0 +1,110 @@
+"""Block attention kernels against the fp64 oracle (Eq. 5, inference mask):
+max-abs 1e-5 for fp32 inputs, 2e-2 for bf16 inputs with fp32 accumulation.
+Cache slots past each sequence's length hold NaN, so any read of them that
+reaches the result fails the comparison."""
+import numpy as np
+import pytest
+
+import gen
+import oracle
+from tests.helpers import BF16_ATTN_TOL, F32_ATTN_TOL, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def sbd():
+    import paper_2509_04185_gb300 as m
+    return m
+
+
+def _run_and_compare(sbd, w, seed=0, num_splits=0, lens=None, scale=0.0):
+    import torch
+    d = gen.attention_inputs(w, seed, poison_tail=lens is None)
+    if lens is not None:
+        d = dict(d)
+        d["cache_len"] = np.asarray(lens, dtype=np.int32)
+        nanv = gen.BF16_NAN if w.dtype == "bf16" else np.float32("nan")
+        for b in range(w.batch):
+            d["k_cache"][b, lens[b]:] = nanv
+            d["v_cache"][b, lens[b]:] = nanv
+    dt = w.dtype
+    args = [to_dev(d[x], dt) for x in ("q", "k_cache", "v_cache")]
+    lens_t = torch.from_numpy(d["cache_len"]).cuda()
+    out = sbd.sbd_block_attention(args[0], args[1], args[2], lens_t, to_dev(d["k_blk"], dt),
+                                  to_dev(d["v_blk"], dt), num_splits=num_splits, scale=scale)
+    got = out.float().cpu().numpy()
+    f = {x: oracle.widen(d[x], dt) for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    ref = oracle.block_attention(f["q"], f["k_cache"], f["v_cache"], d["cache_len"], f["k_blk"],
+                                 f["v_blk"], scale=None if scale == 0.0 else scale)
+    assert np.isfinite(got).all()
+    err = float(np.abs(got - ref).max())
+    tol = F32_ATTN_TOL if dt == "f32" else BF16_ATTN_TOL
+    assert err <= tol, err
+    assert sbd.sbd_device_error() == 0
+    return err
+
+
+def test_tiny_f32_config(sbd):
+    for seed in range(3):
+        _run_and_compare(sbd, gen.get_workload("tiny_f32"), seed)
+
+
+@pytest.mark.parametrize("k,Hq,Hkv", [(1, 4, 2), (3, 8, 2), (7, 4, 4), (32, 2, 2)])
+def test_f32_shapes(sbd, k, Hq, Hkv):
+    w = gen.shrink(gen.get_workload("tiny_f32"), batch=2, block_k=k, n_q_heads=Hq,
+                   n_kv_heads=Hkv, cache_len=(0, 300))
+    _run_and_compare(sbd, w, seed=k)
+
+
+BF16 = gen.get_workload("llama8b_k16")
+
+
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("G,k", [(4, 1), (4, 4), (4, 8), (1, 16), (4, 12), (4, 16), (2, 40 // 2),
+                                 (4, 32), (8, 16)])
+def test_bf16_shapes(sbd, D, G, k):
+    Hkv = 2
+    w = gen.shrink(BF16, batch=2, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv, head_dim=D,
+                   cache_len=(1, 333))
+    _run_and_compare(sbd, w, seed=G * 100 + k)
+
+
+@pytest.mark.parametrize("splits", [1, 2, 3, 7, 40])
+def test_bf16_split_counts(sbd, splits):
+    w = gen.shrink(BF16, batch=3, block_k=16, n_q_heads=8, n_kv_heads=2, cache_len=(0, 700))
+    _run_and_compare(sbd, w, seed=splits, num_splits=splits)
+
+
+def test_bf16_ragged_edges(sbd):
+    # lengths 0, 1, a full tile, a tile + 1 and the maximum
+    w = gen.shrink(BF16, batch=5, block_k=8, n_q_heads=8, n_kv_heads=2, cache_len=(0, 129))
+    _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=2)
+    _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=1)
+
+
+def test_bf16_scale_override(sbd):
+    w = gen.shrink(BF16, batch=1, block_k=4, n_q_heads=8, n_kv_heads=2, cache_len=100)
+    _run_and_compare(sbd, w, scale=0.05)
+
+
+def test_cache_len_out_of_range_is_reported(sbd):
+    import torch
+    w = gen.shrink(BF16, batch=1, block_k=4, n_q_heads=8, n_kv_heads=2, cache_len=64)
+    d = gen.attention_inputs(w, 0, poison_tail=False)
+    t = {x: to_dev(d[x], "bf16") for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    lens = torch.tensor([65], dtype=torch.int32, device="cuda")     # > Lmax: clamped
+    sbd.sbd_block_attention(t["q"], t["k_cache"], t["v_cache"], lens, t["k_blk"], t["v_blk"])
+    assert sbd.sbd_device_error() & sbd.SBD_DEVERR_CACHE_LEN
+    assert sbd.sbd_device_error() == 0
+
+
+@pytest.mark.parametrize("name", ["llama8b_k16", "ragged_b32_k8", "qwen8b_long_k16"])
+def test_full_size_configs(sbd, name):
+    _run_and_compare(sbd, gen.get_workload(name), seed=0)
+
+
+def test_sweep_layer_k32(sbd):
+    """One layer of the 32-layer sweep at its largest block (k = 32: 128
+    packed rows per KV head), batch 16, cache 8192."""
+    _run_and_compare(sbd, gen.sweep_workload(32), seed=0)

@@ -1,0 +1,82 @@
+"""The whole block step loop (Algorithm 3): attention -> LM head with
+entropy and Gumbel-max sampling -> EB select, repeated until the block has
+no masks.  At every step the oracle evaluates the same state; unmask sets
+must match except for the exemptions of the comparison rules."""
+import numpy as np
+import pytest
+
+import gen
+import oracle
+from tests.helpers import ENTROPY_TOL, compare_unmask, step_inputs, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def sbd():
+    import paper_2509_04185_gb300 as m
+    return m
+
+
+def _loop(sbd, w, gamma, seed=0, max_steps=None):
+    import torch
+    d = step_inputs(w, seed)
+    dt = w.dtype
+    att = {x: to_dev(d[x], dt) for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    lens = torch.from_numpy(d["cache_len"]).cuda()
+    W = to_dev(d["w"], dt)
+    masked = torch.from_numpy(d["masked"]).cuda()
+    bt = torch.from_numpy(d["block_tokens"]).cuda()
+    m_host = d["masked"].copy()
+    steps, exempt = 0, 0
+    while m_host.any():
+        sbd.sbd_block_attention(att["q"], att["k_cache"], att["v_cache"], lens, att["k_blk"],
+                                att["v_blk"])
+        hidden = gen.hidden_states(w, seed, steps)
+        gumbel = gen.gumbel_noise(w, seed, steps)
+        ent, tok = sbd.sbd_head_entropy_sample(to_dev(hidden, dt), W, masked,
+                                               torch.from_numpy(gumbel).cuda(), 1.0)
+        n_un = sbd.sbd_eb_select(ent, tok, gamma, masked, bt)
+        new_m = masked.cpu().numpy()
+        # oracle on the same state
+        rent, rtok, _ = oracle.head_entropy_sample(oracle.widen(hidden, dt), d["w"], dt, m_host,
+                                                   gumbel, 1.0)
+        e = ent.cpu().numpy()
+        sel = m_host.astype(bool)
+        assert np.abs(e[sel] - rent[sel]).max() <= ENTROPY_TOL
+        exempt += compare_unmask(m_host, rent, gamma, new_m, tie_tol=2 * ENTROPY_TOL)
+        nu = n_un.cpu().numpy()
+        assert np.all(nu[m_host.any(axis=1)] >= 1)
+        assert np.array_equal(nu, (m_host.astype(int) - new_m.astype(int)).sum(axis=1))
+        m_host = new_m
+        steps += 1
+        assert steps <= w.block_k
+    final = bt.cpu().numpy()
+    assert (final >= 0).all() and (final < w.vocab).all()
+    assert sbd.sbd_device_error() == 0
+    return steps, exempt
+
+
+@pytest.mark.parametrize("gamma", [0.0, 0.1, 1.0])
+def test_tiny_f32_loop(sbd, gamma):
+    w = gen.get_workload("tiny_f32")
+    steps, exempt = _loop(sbd, w, gamma)
+    assert exempt == 0
+    assert 1 <= steps <= 3
+
+
+@pytest.mark.parametrize("gamma", [0.01, 0.1, 1.0])
+def test_llama_small_vocab_loop(sbd, gamma):
+    w = gen.shrink(gen.get_workload("llama8b_k16"), vocab=4096, cache_len=512)
+    steps, exempt = _loop(sbd, w, gamma)
+    assert exempt <= 1
+
+
+def test_llama8b_full_loop(sbd):
+    steps, exempt = _loop(sbd, gen.get_workload("llama8b_k16"), 0.1)
+    assert exempt <= 1
+
+
+def test_ragged_full_loop(sbd):
+    steps, exempt = _loop(sbd, gen.get_workload("ragged_b32_k8"), 0.1)
+    assert exempt <= 2
