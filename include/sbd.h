@@ -126,6 +126,34 @@ sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden
                                    size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * No-allocation variant of sbd_head_entropy_sample.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory -- a host framework that owns the whole device memory pool,
+ * a latency-critical loop that cannot afford the device synchronisation of
+ * cudaMalloc/cudaFree, or a plug-in with no allocator to borrow a workspace
+ * from.  Same arguments, semantics and results as sbd_head_entropy_sample,
+ * minus the workspace: the scratch is a fixed array inside the library, of
+ * SBD_HEAD_NOALLOC_MAX_SCRATCH bytes, which every GPU that loads the library
+ * holds until the process exits.
+ *   - Shapes whose scratch (sbd_head_entropy_sample_workspace_size) exceeds
+ *     that size are rejected with SBD_ERR_UNSUPPORTED before any launch.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first
+ *     call before any stream capture on that device.
+ *   - All calls on a device share the one array, which keeps the last
+ *     call's contents (nothing in it needs to start at zero).  Calls whose
+ *     kernels overlap on the GPU -- on different streams, or from several
+ *     host threads -- race on it: serialise them (one stream, or events).
+ *   - Allocates nothing: no cudaMalloc/cudaFree or allocating library call.
+ * ---------------------------------------------------------------------- */
+#define SBD_HEAD_NOALLOC_MAX_SCRATCH (4u << 20) /* 4 MiB */
+
+sbd_status sbd_head_entropy_sample_noalloc(const sbd_head_desc* desc, const void* hidden,
+                                           const void* w, const uint8_t* masked,
+                                           const float* gumbel, float tau, float* entropy,
+                                           int32_t* token, void* stream);
+
+/* ------------------------------------------------------------------------
  * Entropy-bounded select, entropy proxy (Eq. 3; Algorithm 3 "unmask").  Per
  * sequence b: sort the masked positions by (entropy, position) ascending,
  * i_1, i_2, ...; accept the first s >= 1 positions, s the largest value with

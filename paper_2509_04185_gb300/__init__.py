@@ -32,6 +32,7 @@ SBD_DTYPE_BF16 = 1
 SBD_DEVERR_CACHE_LEN = 1
 SBD_DEVERR_TIMEOUT = 2
 SBD_DEVERR_ROWS = 4
+SBD_HEAD_NOALLOC_MAX_SCRATCH = 4 << 20
 
 # Every symbol include/sbd.h declares.
 EXPORTS = (
@@ -39,6 +40,7 @@ EXPORTS = (
     "sbd_block_attention",
     "sbd_head_entropy_sample_workspace_size",
     "sbd_head_entropy_sample",
+    "sbd_head_entropy_sample_noalloc",
     "sbd_eb_select",
     "sbd_status_string",
     "sbd_last_error",
@@ -82,6 +84,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_head_entropy_sample.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp, f32, vp,
                                             vp, vp, sz, vp]
     lib.sbd_head_entropy_sample.restype = ctypes.c_int
+    lib.sbd_head_entropy_sample_noalloc.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp,
+                                                    f32, vp, vp, vp]
+    lib.sbd_head_entropy_sample_noalloc.restype = ctypes.c_int
     lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
     lib.sbd_eb_select.restype = ctypes.c_int
     lib.sbd_status_string.argtypes = [ctypes.c_int]
@@ -210,6 +215,24 @@ def sbd_head_entropy_sample(hidden, w, masked, gumbel, tau: float, entropy=None,
     _check(lib.sbd_head_entropy_sample(ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked),
                                        _ptr(gumbel), float(tau), _ptr(entropy), _ptr(token),
                                        _ptr(ws), _nbytes(ws), _stream(stream)))
+    return entropy, token
+
+
+def sbd_head_entropy_sample_noalloc(hidden, w, masked, gumbel, tau: float, entropy, token, *,
+                                    stream=None):
+    """sbd_head_entropy_sample for callers that cannot allocate device
+    memory: the scratch is the library's fixed device array (shared by every
+    call on a device; calls must not overlap on the GPU).  The outputs
+    entropy [B,k] fp32 and token [B,k] int32 are caller-provided; nothing is
+    allocated here or in the library."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, gumbel=gumbel, entropy=entropy, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    d = head_desc(hidden, w)
+    _check(lib.sbd_head_entropy_sample_noalloc(ctypes.byref(d), _ptr(hidden), _ptr(w),
+                                               _ptr(masked), _ptr(gumbel), float(tau),
+                                               _ptr(entropy), _ptr(token), _stream(stream)))
     return entropy, token
 
 
