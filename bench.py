@@ -218,20 +218,24 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
     gamma, tau = args.gamma, args.tau
 
+    attn_call = sbd.prepare_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"],
+                                            T["k_blk"], T["v_blk"], out, ws_a, stream=stream)
+    head_call = sbd.prepare_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau,
+                                                ent, tok, ws_h, stream=stream)
+    eb_call = sbd.prepare_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
+
     def step(ev=None):
         masked.copy_(masked0, non_blocking=True)
         bt.copy_(bt0, non_blocking=True)
         if ev is not None:
             ev[0].record(stream)
-        sbd.sbd_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"], T["k_blk"],
-                                T["v_blk"], out, workspace=ws_a, stream=stream)
+        attn_call()
         if ev is not None:
             ev[1].record(stream)
-        sbd.sbd_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau, ent, tok,
-                                    workspace=ws_h, stream=stream)
+        head_call()
         if ev is not None:
             ev[2].record(stream)
-        sbd.sbd_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
+        eb_call()
         if ev is not None:
             ev[3].record(stream)
 
@@ -294,11 +298,9 @@ def run_ours(args):
                 T[k].copy_(host[k], non_blocking=True)
             masked.copy_(host["masked"], non_blocking=True)
             bt.copy_(host["block_tokens"], non_blocking=True)
-            sbd.sbd_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"],
-                                    T["k_blk"], T["v_blk"], out, workspace=ws_a, stream=stream)
-            sbd.sbd_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau, ent, tok,
-                                        workspace=ws_h, stream=stream)
-            sbd.sbd_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
+            attn_call()
+            head_call()
+            eb_call()
             res["out"].copy_(out, non_blocking=True)
             res["ent"].copy_(ent, non_blocking=True)
             res["tok"].copy_(tok, non_blocking=True)
@@ -486,6 +488,180 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------------ sweep
+
+def run_sweep(args):
+    """The 32-layer block-step loop at Llama-3.1-8B attention shapes
+    (Algorithm 3): every block starts fully masked; each step runs block
+    attention over all 32 layers' KV caches, the LM head with entropy and
+    Gumbel-max sampling over the still-masked positions, and the EB select;
+    steps repeat until no position of any sequence is masked (one 4-byte
+    read of the remaining count per step).  A timed step is one such
+    iteration; the timed region covers whole blocks.
+
+    The 17 GB of per-layer caches and the other large inputs are drawn on the
+    device with PyTorch's seeded generator (the parity tests use the host
+    generator on one layer of the same shapes).  Hidden rows are redrawn per
+    step; the Gumbel noise of a block is drawn once and indexed by block
+    position, so each committed token is a Gumbel-max sample at its commit
+    step."""
+    import torch
+
+    import paper_2509_04185_gb300 as sbd
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = gen.get_workload(args.workload)
+    B, k, Hq, Hkv, D, L = w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim, w.max_cache_len
+    V, H, NL = w.vocab, w.hidden, w.n_layers
+    g = torch.Generator(device=dev)
+    g.manual_seed(args.seed * 1000003 + 17)
+
+    def randn(*shape, std=1.0):
+        return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32) * std).bfloat16()
+
+    layers = []
+    for _ in range(NL):
+        layers.append(dict(q=randn(B, k, Hq, D), kc=randn(B, L, Hkv, D), vc=randn(B, L, Hkv, D),
+                           kb=randn(B, k, Hkv, D), vb=randn(B, k, Hkv, D)))
+    lens = torch.full((B,), L, dtype=torch.int32, device=dev)
+    Wt = randn(V, H, std=w.w_std)
+    lo, hi = np.log(w.hidden_scale[0]), np.log(w.hidden_scale[1])
+    hidden = []
+    for _ in range(k):
+        h = torch.randn(B, k, H, generator=g, device=dev)
+        sc = torch.exp(torch.empty(B, k, 1, device=dev).uniform_(lo, hi, generator=g))
+        hidden.append((h * sc).bfloat16())
+    u = torch.rand(B, k, V, generator=g, device=dev, dtype=torch.float64).clamp_(1e-300, 1 - 1e-16)
+    gumbel = (-torch.log(-torch.log(u))).float()
+    del u
+    outs = [torch.empty_like(layers[0]["q"]) for _ in range(NL)]
+    masked = torch.ones(B, k, dtype=torch.uint8, device=dev)
+    bt = torch.full((B, k), -1, dtype=torch.int32, device=dev)
+    ent = torch.empty(B, k, dtype=torch.float32, device=dev)
+    tok = torch.empty(B, k, dtype=torch.int32, device=dev)
+    n_un = torch.empty(B, dtype=torch.int32, device=dev)
+    left_h = torch.empty(1, dtype=torch.int32).pin_memory()
+    stream = torch.cuda.current_stream(dev)
+    import ctypes
+    ad = sbd.attn_desc(layers[0]["q"], layers[0]["kc"])
+    ws_a = torch.empty(max(1, sbd.lib.sbd_block_attention_workspace_size(ctypes.byref(ad))),
+                       dtype=torch.uint8, device=dev)
+    hd = sbd.head_desc(hidden[0], Wt)
+    ws_h = torch.empty(max(1, sbd.lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(hd))),
+                       dtype=torch.uint8, device=dev)
+    attn_calls = [sbd.prepare_block_attention(L_["q"], L_["kc"], L_["vc"], lens, L_["kb"], L_["vb"],
+                                              outs[i], ws_a, stream=stream)
+                  for i, L_ in enumerate(layers)]
+    head_calls = [sbd.prepare_head_entropy_sample(hidden[s_], Wt, masked, gumbel, args.tau, ent, tok,
+                                                  ws_h, stream=stream) for s_ in range(k)]
+    eb_call = sbd.prepare_eb_select(ent, tok, args.gamma, masked, bt, n_un, stream=stream)
+
+    def block(ev=None):
+        """One block: steps until no masks.  Returns the step count."""
+        masked.fill_(1)
+        bt.fill_(-1)
+        steps = 0
+        while True:
+            if ev is not None:
+                ev.append([torch.cuda.Event(enable_timing=True) for _ in range(4)])
+                ev[-1][0].record(stream)
+            for c in attn_calls:
+                c()
+            if ev is not None:
+                ev[-1][1].record(stream)
+            head_calls[min(steps, k - 1)]()
+            if ev is not None:
+                ev[-1][2].record(stream)
+            eb_call()
+            if ev is not None:
+                ev[-1][3].record(stream)
+            left_h.copy_(masked.sum(dtype=torch.int32).view(1), non_blocking=True)
+            stream.synchronize()
+            steps += 1
+            if int(left_h.item()) == 0 or steps >= k:
+                return steps
+
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    for _ in range(max(1, args.warmup // max(1, k // 2))):
+        block()
+    torch.cuda.synchronize(dev)
+    if sbd.sbd_device_error() != 0:
+        raise RuntimeError("device error word set during warm-up")
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    if sampler:
+        sampler.mark("timed_start")
+    evs = []
+    t0 = time.perf_counter()
+    n_steps, n_blocks = 0, 0
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    while n_steps < args.steps:
+        n_steps += block(evs)
+        n_blocks += 1
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - t0
+    if sampler:
+        sampler.mark("timed_end")
+    total_ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.barrier()
+        total_ms = float(t.item())
+    attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    if sbd.sbd_device_error() != 0:
+        raise RuntimeError("device error word set during the timed region")
+    clocks = sampler.stop() if sampler else None
+    if rank != 0:
+        return
+    peaks, peak_src = measured_peaks()
+    e = 2
+    attn_bytes = NL * (2 * B * L * Hkv * D + 2 * B * k * Hkv * D + 2 * B * k * Hq * D) * e
+    # masked rows average over the steps of a block: k rows at the first step
+    head_bytes_first = V * H * e + B * k * H * e + B * k * V * 4
+    ms_per_step = total_ms / n_steps
+    attn_gbs = attn_bytes / (attn_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": round(ms_per_step * 1000.0 / world, 3), "unit": UNIT,
+        "n_gpus": world, "steps": n_steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 6), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (PyTorch seeded device generator; random-init LM head)",
+        "config": {"workload": args.workload, "batch": B, "block_k": k, "layers": NL,
+                   "cache_len": L, "hidden": H, "vocab": V, "gamma": args.gamma, "tau": args.tau,
+                   "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2: 17 GB of KV caches per step"},
+        "steps_per_block": round(n_steps / n_blocks, 3),
+        "blocks": n_blocks,
+        "tokens_committed_per_s": round(n_blocks * B * k / (total_ms * 1e-3) * world, 1),
+        "gpu_launches": int(n_steps * (NL * (2 if ws_a.numel() > 1 else 1) + 3 + 1)),
+        "per_call_us": {"attention_32_layers": round(attn_ms * 1000, 3),
+                        "head": round(head_ms * 1000, 3), "eb_select": round(eb_ms * 1000, 3)},
+        "roofline": {
+            "kernel": "block attention, 32 layers (attn_bf16_kernel + split combine)",
+            "bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"],
+            "peak_source": peak_src, "unit": "GB/s", "frac": round(attn_gbs / peaks["hbm_gbs"], 4),
+            "traffic": None, "algorithmic_bytes": int(attn_bytes)},
+        "head_first_step_bytes": int(head_bytes_first),
+        "host_wall_s": round(wall, 3),
+        "clocks": clocks, "e2e": None, "cpu_baseline": None,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -493,7 +669,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b_k16",
-                    choices=["llama8b_k16", "ragged_b32_k8", "qwen8b_long_k16", "tiny_f32"])
+                    choices=["llama8b_k16", "ragged_b32_k8", "qwen8b_long_k16", "tiny_f32",
+                             "sweep32_k4", "sweep32_k8", "sweep32_k16", "sweep32_k32"])
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--gamma", type=float, default=0.1)
     ap.add_argument("--tau", type=float, default=1.0)
@@ -504,6 +681,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload.startswith("sweep32"):
+        run_sweep(args)
     else:
         run_ours(args)
 

@@ -106,7 +106,7 @@ sbd_status sbd_block_attention(const sbd_attn_desc* desc, const void* q,
  *   gumbel [B, k, V] fp32, indexed by block position; may be NULL iff
  *          tau == 0 (greedy); rows of unmasked positions are not read
  *   entropy [B, k] fp32 out, token [B, k] int32 out
- * Supported: B * k <= 256, H % 64 == 0 for bf16 (H % 4 == 0 for fp32),
+ * Supported: B * k <= 512, H % 64 == 0 for bf16 (H % 4 == 0 for fp32),
  * tau >= 0 and finite.
  * ---------------------------------------------------------------------- */
 typedef struct {

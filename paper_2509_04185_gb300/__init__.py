@@ -251,6 +251,67 @@ def sbd_eb_select(entropy, token, gamma: float, masked, block_tokens, n_unmasked
     return n_unmasked
 
 
+class Prepared:
+    """A library call with every argument already marshalled: calling it
+    re-issues the same C call (same tensors, stream and workspace) with no
+    Python-side checks.  For step loops that repeat one call shape."""
+
+    __slots__ = ("_fn", "_args", "_keep")
+
+    def __init__(self, fn, args, keep):
+        self._fn = fn
+        self._args = args
+        self._keep = keep          # tensors whose memory the pointers refer to
+
+    def __call__(self) -> None:
+        st = self._fn(*self._args)
+        if st != SBD_OK:
+            raise SbdError(st, lib.sbd_last_error().decode())
+
+
+def prepare_block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, out, workspace=None,
+                            *, scale: float = 0.0, num_splits: int = 0, stream=None) -> Prepared:
+    """sbd_block_attention bound to fixed tensors (see Prepared)."""
+    torch = _torch()
+    _need_cuda(q=q, k_cache=k_cache, v_cache=v_cache, cache_len=cache_len, k_blk=k_blk,
+               v_blk=v_blk, out=out)
+    if cache_len.dtype != torch.int32:
+        raise TypeError("cache_len must be int32")
+    d = attn_desc(q, k_cache, scale, num_splits)
+    ws = _workspace(lib.sbd_block_attention_workspace_size(ctypes.byref(d)), q.device, workspace)
+    args = (ctypes.byref(d), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(k_blk),
+            _ptr(v_blk), _ptr(out), _ptr(ws), _nbytes(ws), _stream(stream))
+    return Prepared(lib.sbd_block_attention, args,
+                    (d, q, k_cache, v_cache, cache_len, k_blk, v_blk, out, ws))
+
+
+def prepare_head_entropy_sample(hidden, w, masked, gumbel, tau: float, entropy, token,
+                                workspace=None, *, stream=None) -> Prepared:
+    """sbd_head_entropy_sample bound to fixed tensors (see Prepared)."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, gumbel=gumbel, entropy=entropy, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    d = head_desc(hidden, w)
+    ws = _workspace(lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(d)), hidden.device,
+                    workspace)
+    args = (ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked), _ptr(gumbel), float(tau),
+            _ptr(entropy), _ptr(token), _ptr(ws), _nbytes(ws), _stream(stream))
+    return Prepared(lib.sbd_head_entropy_sample, args,
+                    (d, hidden, w, masked, gumbel, entropy, token, ws))
+
+
+def prepare_eb_select(entropy, token, gamma: float, masked, block_tokens, n_unmasked, *,
+                      stream=None) -> Prepared:
+    """sbd_eb_select bound to fixed tensors (see Prepared)."""
+    _need_cuda(entropy=entropy, token=token, masked=masked, block_tokens=block_tokens,
+               n_unmasked=n_unmasked)
+    B, k = masked.shape
+    args = (B, k, _ptr(entropy), _ptr(token), float(gamma), _ptr(masked), _ptr(block_tokens),
+            _ptr(n_unmasked), _stream(stream))
+    return Prepared(lib.sbd_eb_select, args, (entropy, token, masked, block_tokens, n_unmasked))
+
+
 def sbd_device_error() -> int:
     """Reads and clears the device error word (synchronises the device)."""
     code = ctypes.c_int32(0)

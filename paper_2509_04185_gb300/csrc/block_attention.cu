@@ -30,7 +30,20 @@ namespace {
 using namespace sbd_dev;
 
 constexpr int kTileKeys = 64;
-constexpr int kStages = 4;
+constexpr int kMaxStages = 4;
+// Ring depth cap and the key-group count used for 4 row tiles (64 packed
+// rows); defaults chosen by measurement.
+#ifndef SBD_ATTN_STAGE_CAP
+#define SBD_ATTN_STAGE_CAP 3
+#endif
+#ifndef SBD_ATTN_KG_MT4
+#define SBD_ATTN_KG_MT4 1
+#endif
+// bf16 attention on the tcgen05 kernel (block_attention_tc.cu) rather than
+// the mma.sync kernel of this file.
+#ifndef SBD_ATTN_TC
+#define SBD_ATTN_TC 1
+#endif
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------ mma helpers
@@ -75,12 +88,12 @@ struct AttnArgs {
   float* part_o;             // [B, Hkv, S, M, D] (splits > 1)
   float* part_lse;           // [B, Hkv, S, M]
   int* err;
-  int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG;
+  int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG, stages;
   float scale_log2;
 };
 
-template <int D>
-__global__ void __launch_bounds__(288, 1)
+template <int D, int NK>
+__global__ void __launch_bounds__(288)
 attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
                  const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
   constexpr int kSub = D / 64;                       // 128-B column sub-tiles per row
@@ -88,18 +101,31 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
   constexpr int kStageBytes = 2 * kSub * kSubBytes;  // K then V
   constexpr int kDT = D / 8;                         // n-tiles of the output
   constexpr int kKS = D / 16;                        // k-steps of Q K^T
+  constexpr int kNT = NK / 8;                        // score n-tiles per warp and tile
 
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kStages];
-  __shared__ __align__(8) uint64_t empty_bar[kStages];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
 
   const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* smem_gen = smem_raw + (smem_base - smem_u32(smem_raw));
-  float* merge_buf = reinterpret_cast<float*>(smem_gen + kStages * kStageBytes);
+  // The key-group merge reuses the ring once every tile has been consumed.
+  float* merge_buf = reinterpret_cast<float*>(smem_gen);
+  const int kStages = a.stages;
 
   const int NW = a.MT * a.KG;                        // compute warps
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], NW);
+    }
+    fence_mbar_init();
+  }
+  // Everything below may read what the previous kernel on the stream wrote.
+  grid_dependency_wait();
 
   int len = a.lens[b];
   if (len < 0 || len > a.Lmax) {
@@ -110,14 +136,6 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const int n_tiles = n_cache_tiles + 1;             // + the block tile
   const int t_begin = (int)((long long)split * n_tiles / a.splits);
   const int t_end = (int)((long long)(split + 1) * n_tiles / a.splits);
-
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full_bar[s], 1);
-      mbar_init(&empty_bar[s], NW);
-    }
-    fence_mbar_init();
-  }
   __syncthreads();
 
   if (warp == NW) {
@@ -177,8 +195,7 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
   } else if (warp < NW) {
     // ------------------------------------------------ compute warps
-    const int rt = warp % a.MT, kg = warp / a.MT;
-    const int NK = kTileKeys / a.KG;                 // keys of a tile handled by this warp
+    const int rt = warp % a.MT, kg = warp / a.MT;    // NK keys of each tile per warp
     const int r0 = rt * 16 + (lane >> 2), r1 = r0 + 8;
     const int qc = (lane & 3) * 2;
 
@@ -224,72 +241,81 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
       const uint32_t vbase = kbase + kSub * kSubBytes;
       const int key0 = kg * NK;
 
-      // Process this warp's NK keys in chunks of 16 keys.
-      for (int kc = 0; kc < NK; kc += 16) {
-        const int j0 = key0 + kc;
-        float s[2][4];
+      // S = Q K^T over this warp's NK keys of the tile: NK/8 independent
+      // accumulators per k-step.
+      float s[kNT][4];
 #pragma unroll
-        for (int n = 0; n < 2; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+      for (int n = 0; n < kNT; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
 #pragma unroll
-        for (int ks = 0; ks < kKS; ++ks) {
-          const int key = j0 + ((lm >= 2) ? 8 : 0) + lr;
+      for (int ks = 0; ks < kKS; ++ks) {
+#pragma unroll
+        for (int np = 0; np < NK / 16; ++np) {
+          const int key = key0 + np * 16 + ((lm >= 2) ? 8 : 0) + lr;
           const int d = ks * 16 + ((lm & 1) ? 8 : 0);
           uint32_t b0, b1, b2, b3;
           ldsm_x4(swz(kbase + (d >> 6) * kSubBytes, key, (d & 63) >> 3), b0, b1, b2, b3);
-          mma_bf16(s[0], qa[ks], b0, b1);
-          mma_bf16(s[1], qa[ks], b2, b3);
+          mma_bf16(s[2 * np], qa[ks], b0, b1);
+          mma_bf16(s[2 * np + 1], qa[ks], b2, b3);
         }
-        // scale + mask in registers
-        float mx0 = -INFINITY, mx1 = -INFINITY;
+      }
+      // scale + mask in registers, then one online-softmax update per tile
+      float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-        for (int n = 0; n < 2; ++n) {
+      for (int n = 0; n < kNT; ++n) {
 #pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int key = j0 + n * 8 + qc + e;
-            const bool vis = key < valid;
-            s[n][e] = vis ? s[n][e] * a.scale_log2 : -INFINITY;
-            s[n][2 + e] = vis ? s[n][2 + e] * a.scale_log2 : -INFINITY;
-            mx0 = fmaxf(mx0, s[n][e]);
-            mx1 = fmaxf(mx1, s[n][2 + e]);
-          }
+        for (int e = 0; e < 2; ++e) {
+          const int key = key0 + n * 8 + qc + e;
+          const bool vis = key < valid;
+          s[n][e] = vis ? s[n][e] * a.scale_log2 : -INFINITY;
+          s[n][2 + e] = vis ? s[n][2 + e] * a.scale_log2 : -INFINITY;
+          mx0 = fmaxf(mx0, s[n][e]);
+          mx1 = fmaxf(mx1, s[n][2 + e]);
         }
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        const float mu0 = (mn0 == -INFINITY) ? 0.f : mn0;
-        const float mu1 = (mn1 == -INFINITY) ? 0.f : mn1;
-        const float al0 = exp2f(m0 - mu0), al1 = exp2f(m1 - mu1);
-        m0 = mn0;
-        m1 = mn1;
-        float ps0 = 0.f, ps1 = 0.f;
+      }
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float mu0 = (mn0 == -INFINITY) ? 0.f : mn0;
+      const float mu1 = (mn1 == -INFINITY) ? 0.f : mn1;
+      const float al0 = exp2f(m0 - mu0), al1 = exp2f(m1 - mu1);
+      m0 = mn0;
+      m1 = mn1;
+      float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
-        for (int n = 0; n < 2; ++n) {
-          s[n][0] = exp2f(s[n][0] - mu0);
-          s[n][1] = exp2f(s[n][1] - mu0);
-          s[n][2] = exp2f(s[n][2] - mu1);
-          s[n][3] = exp2f(s[n][3] - mu1);
-          ps0 += s[n][0] + s[n][1];
-          ps1 += s[n][2] + s[n][3];
-        }
-        l0 = l0 * al0 + ps0;
-        l1 = l1 * al1 + ps1;
+      for (int n = 0; n < kNT; ++n) {
+        s[n][0] = exp2f(s[n][0] - mu0);
+        s[n][1] = exp2f(s[n][1] - mu0);
+        s[n][2] = exp2f(s[n][2] - mu1);
+        s[n][3] = exp2f(s[n][3] - mu1);
+        ps0 += s[n][0] + s[n][1];
+        ps1 += s[n][2] + s[n][3];
+      }
+      l0 = l0 * al0 + ps0;
+      l1 = l1 * al1 + ps1;
 #pragma unroll
-        for (int i = 0; i < kDT; ++i) {
-          o[i][0] *= al0;
-          o[i][1] *= al0;
-          o[i][2] *= al1;
-          o[i][3] *= al1;
-        }
+      for (int i = 0; i < kDT; ++i) {
+        o[i][0] *= al0;
+        o[i][1] *= al0;
+        o[i][2] *= al1;
+        o[i][3] *= al1;
+      }
+      // O += P V, 16 keys per k-step.  Value rows past `valid` are zeroed in
+      // registers so that unused cache slots (possibly NaN) never meet a zero
+      // probability.
+#pragma unroll
+      for (int kk = 0; kk < NK / 16; ++kk) {
+        const int j0 = key0 + kk * 16;
         uint32_t pa[4];
-        pa[0] = pack_bf16(s[0][0], s[0][1]);
-        pa[1] = pack_bf16(s[0][2], s[0][3]);
-        pa[2] = pack_bf16(s[1][0], s[1][1]);
-        pa[3] = pack_bf16(s[1][2], s[1][3]);
-        // V fragments (trans), keys j0..j0+15; zero keys past `valid` so that
-        // unused cache slots (possibly NaN) never meet a zero probability.
+        pa[0] = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
+        pa[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
+        pa[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+        pa[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
         const bool sanitize = j0 + 16 > valid;
+        const int ka = j0 + qc, kb8 = j0 + 8 + qc;
+        const uint32_t m_a = (ka < valid ? 0xffffu : 0u) | (ka + 1 < valid ? 0xffff0000u : 0u);
+        const uint32_t m_b = (kb8 < valid ? 0xffffu : 0u) | (kb8 + 1 < valid ? 0xffff0000u : 0u);
 #pragma unroll
         for (int dp = 0; dp < kDT / 2; ++dp) {
           const int key = j0 + ((lm & 1) ? 8 : 0) + lr;
@@ -297,10 +323,6 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
           uint32_t b0, b1, b2, b3;
           ldsm_x4_t(swz(vbase + (d >> 6) * kSubBytes, key, (d & 63) >> 3), b0, b1, b2, b3);
           if (sanitize) {
-            const int ka = j0 + qc, kb8 = j0 + 8 + qc;
-            const uint32_t m_a = (ka < valid ? 0xffffu : 0u) | (ka + 1 < valid ? 0xffff0000u : 0u);
-            const uint32_t m_b =
-                (kb8 < valid ? 0xffffu : 0u) | (kb8 + 1 < valid ? 0xffff0000u : 0u);
             b0 &= m_a;
             b1 &= m_b;
             b2 &= m_a;
@@ -314,6 +336,7 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
       if (lane == 0) mbar_arrive(&empty_bar[stage]);
     }
     (void)ok;
+    grid_dependents_launch();
 
     // Row sums across the 4 threads of a row.
     l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
@@ -325,6 +348,8 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
     if (a.KG > 1) {
       // layout per warp: [16 rows][D] o, then [16] m, [16] l
       float* mine = merge_buf + warp * (16 * D + 32);
+      // every compute warp is done reading the ring before it is reused
+      asm volatile("bar.sync 1, %0;" ::"r"(NW * 32) : "memory");
       if (kg > 0) {
 #pragma unroll
         for (int i = 0; i < kDT; ++i) {
@@ -410,40 +435,45 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
   }
 }
 
-// Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.
+// Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.  One CTA per
+// (packed row, KV head, sequence); thread d owns output element d.
 template <typename OutT>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(128)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
-                    OutT* __restrict__ out, int B, int k, int Hq, int Hkv, int G, int M, int D,
+                    OutT* __restrict__ out, int k, int Hq, int Hkv, int G, int M, int D,
                     int splits) {
-  extern __shared__ float wsm[];                     // [splits][M] weights, then [M] 1/sum
-  const int pair = blockIdx.x;                       // b * Hkv + hkv
-  const int b = pair / Hkv, hkv = pair % Hkv;
-  const float* lse = part_lse + (size_t)pair * splits * M;
-  const float* po = part_o + (size_t)pair * splits * M * D;
-  for (int r = threadIdx.x; r < M; r += blockDim.x) {
+  __shared__ float w_s[64];
+  __shared__ float inv_sum;
+  grid_dependency_wait();
+  const int r = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+  const size_t pair = (size_t)b * Hkv + hkv;
+  const float* lse = part_lse + pair * splits * M;
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
     float mx = -INFINITY;
-    for (int s = 0; s < splits; ++s) mx = fmaxf(mx, lse[s * M + r]);
+    for (int s = lane; s < splits; s += 32) mx = fmaxf(mx, lse[(size_t)s * M + r]);
+    mx = warp_max(mx);
     float sum = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      const float w = (mx == -INFINITY) ? 0.f : exp2f(lse[s * M + r] - mx);
-      wsm[s * M + r] = w;
-      sum += w;
+    for (int s = lane; s < splits; s += 32) {
+      const float wt = (mx == -INFINITY) ? 0.f : exp2f(lse[(size_t)s * M + r] - mx);
+      w_s[s] = wt;
+      sum += wt;
     }
-    wsm[splits * M + r] = sum > 0.f ? 1.f / sum : 0.f;
+    sum = warp_sum(sum);
+    if (lane == 0) inv_sum = sum > 0.f ? 1.f / sum : 0.f;
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < M * D; e += blockDim.x) {
-    const int r = e / D, d = e % D;
-    float acc = 0.f;
-    for (int s = 0; s < splits; ++s) acc += wsm[s * M + r] * po[((size_t)s * M + r) * D + d];
-    acc *= wsm[splits * M + r];
-    const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + d;
-    if constexpr (sizeof(OutT) == 2)
-      out[o] = __float2bfloat16_rn(acc);
-    else
-      out[o] = acc;
-  }
+  const int d = threadIdx.x;
+  if (d >= D) return;
+  const float* po = part_o + (pair * splits * M + r) * D + d;
+  float acc = 0.f;
+  for (int s = 0; s < splits; ++s) acc += w_s[s] * po[(size_t)s * M * D];
+  acc *= inv_sum;
+  const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + d;
+  if constexpr (sizeof(OutT) == 2)
+    out[o] = __float2bfloat16_rn(acc);
+  else
+    out[o] = acc;
 }
 
 // ------------------------------------------------------------ fp32 variant
@@ -454,10 +484,11 @@ attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
                 const float* __restrict__ vc, const int32_t* __restrict__ lens,
                 const float* __restrict__ kb, const float* __restrict__ vb,
                 float* __restrict__ out, int* err, int k, int Hq, int Hkv, int D, int Lmax,
-                float scale_log2, int splits, float* part_o, float* part_lse) {
+                float scale_log2) {
   __shared__ float qs[128];
   __shared__ float ps[128];
   __shared__ float red[4];
+  grid_dependency_wait();
   const int i = blockIdx.x, hq = blockIdx.y, b = blockIdx.z;
   const int G = Hq / Hkv, hkv = hq / G;
   const int tid = threadIdx.x;
@@ -510,9 +541,6 @@ attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
     __syncthreads();
   }
   if (tid < D) out[(((size_t)b * k + i) * Hq + hq) * D + tid] = acc / l;
-  (void)splits;
-  (void)part_o;
-  (void)part_lse;
 }
 
 }  // namespace
@@ -551,14 +579,23 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
   p.bf16 = d.dtype == SBD_DTYPE_BF16;
   const float scale = d.scale != 0.f ? d.scale : 1.0f / sqrtf((float)d.head_dim);
   p.scale_log2 = scale * kLog2e;
+  const int tiles = (p.Lmax + kTileKeys - 1) / kTileKeys + 1;
   if (!p.bf16) {
     p.splits = 1;
   } else if (d.num_splits > 0) {
     p.splits = d.num_splits;
   } else {
-    const int tiles = (p.Lmax + kTileKeys - 1) / kTileKeys + 1;
     p.splits = choose_splits(p.B * p.Hkv, tiles, num_sms());
   }
+  // Ring depth: as many stages as a split has tiles, between 2 and 4.
+  const int per_split = (tiles + p.splits - 1) / p.splits;
+  const int cap = SBD_ATTN_STAGE_CAP < kMaxStages ? SBD_ATTN_STAGE_CAP : kMaxStages;
+  p.stages = per_split < 2 ? 2 : (per_split > cap ? cap : per_split);
+  // Row tiles of 16 packed rows; small tiles also split every key tile
+  // between key groups so that at least 4 (up to 8) warps share the work.
+  p.MT = (p.M + 15) / 16;
+  p.KG = p.MT >= 5 ? 1 : (p.MT == 4 ? SBD_ATTN_KG_MT4 : (p.MT == 3 ? 2 : 4));
+  if (p.MT == 1) p.KG = 4;
   return p;
 }
 
@@ -568,10 +605,10 @@ size_t attn_workspace_bytes(const AttnPlan& p) {
   return align_up(n * p.D * sizeof(float), 256) + align_up(n * sizeof(float), 256);
 }
 
-static size_t attn_smem_bytes(int D, int NW, int KG) {
-  const size_t stages = (size_t)kStages * 2 * (D / 64) * kTileKeys * 128;
-  const size_t merge = KG > 1 ? (size_t)NW * (16 * D + 32) * sizeof(float) : 0;
-  return 1024 + stages + merge;
+static size_t attn_smem_bytes(const AttnPlan& p) {
+  const size_t ring = (size_t)p.stages * 2 * (p.D / 64) * kTileKeys * 128;
+  const size_t merge = p.KG > 1 ? (size_t)p.MT * p.KG * (16 * p.D + 32) * sizeof(float) : 0;
+  return 1024 + (ring > merge ? ring : merge);
 }
 
 sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const void* vc,
@@ -580,13 +617,16 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   if (p.B == 0) return SBD_OK;
   int* err = device_error_word();
   if (!p.bf16) {
-    dim3 grid(p.k, p.Hq, p.B);
-    attn_f32_kernel<<<grid, 128, 0, st>>>(
-        (const float*)q, (const float*)kc, (const float*)vc, lens, (const float*)kb,
-        (const float*)vb, (float*)out, err, p.k, p.Hq, p.Hkv, p.D, p.Lmax, p.scale_log2, 1,
-        nullptr, nullptr);
-    cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? SBD_OK : cuda_fail(e, "attn_f32_kernel launch");
+    const float *qf = (const float*)q, *kcf = (const float*)kc, *vcf = (const float*)vc;
+    const float *kbf = (const float*)kb, *vbf = (const float*)vb;
+    float* of = (float*)out;
+    int k = p.k, Hq = p.Hq, Hkv = p.Hkv, D = p.D, Lmax = p.Lmax;
+    float sl2 = p.scale_log2;
+    void* args[] = {(void*)&qf, (void*)&kcf, (void*)&vcf, (void*)&lens, (void*)&kbf,
+                    (void*)&vbf, (void*)&of,  (void*)&err, (void*)&k,    (void*)&Hq,
+                    (void*)&Hkv, (void*)&D,   (void*)&Lmax, (void*)&sl2};
+    return launch_pdl((const void*)attn_f32_kernel, dim3(p.k, p.Hq, p.B), dim3(128), 0, st, args,
+                      "attn_f32_kernel launch");
   }
 
   // 4-D tensor maps over the caches: dims (D, Hkv, Lmax, B), 64x64 boxes.
@@ -617,38 +657,50 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.M = p.M;
   a.Lmax = p.Lmax;
   a.splits = p.splits;
-  a.MT = (p.M + 15) / 16;
-  a.KG = a.MT >= 4 ? 1 : 4 / a.MT;
+  a.MT = p.MT;
+  a.KG = p.KG;
+  a.stages = p.stages;
   a.scale_log2 = p.scale_log2;
   const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
   a.part_o = (float*)ws;
   a.part_lse = p.splits > 1 ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
 
-  const int NW = a.MT * a.KG;
-  const size_t smem = attn_smem_bytes(p.D, NW, a.KG);
-  dim3 grid(p.splits, p.Hkv, p.B);
-  dim3 block(32 * (NW + 1));
-  cudaError_t e;
-  if (p.D == 128) {
-    e = cudaFuncSetAttribute(attn_bf16_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_bf16_kernel)");
-    attn_bf16_kernel<128><<<grid, block, smem, st>>>(tk, tv, a);
+  // Up to 16 packed rows the mma.sync kernel measures faster (the tcgen05
+  // kernel pads every tile to 128 rows); above, tcgen05.
+  if (SBD_ATTN_TC && p.M > 16) {
+    s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, st);
+    if (s != SBD_OK) return s;
   } else {
-    e = cudaFuncSetAttribute(attn_bf16_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_bf16_kernel)");
-    attn_bf16_kernel<64><<<grid, block, smem, st>>>(tk, tv, a);
+  const int NW = a.MT * a.KG;
+  const size_t smem = attn_smem_bytes(p);
+  const void* fn;
+  if (p.D == 128)
+    fn = p.KG == 1 ? (const void*)attn_bf16_kernel<128, 64>
+                   : (p.KG == 2 ? (const void*)attn_bf16_kernel<128, 32>
+                                : (const void*)attn_bf16_kernel<128, 16>);
+  else
+    fn = p.KG == 1 ? (const void*)attn_bf16_kernel<64, 64>
+                   : (p.KG == 2 ? (const void*)attn_bf16_kernel<64, 32>
+                                : (const void*)attn_bf16_kernel<64, 16>);
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_bf16_kernel)");
+  {
+    void* args[] = {(void*)&tk, (void*)&tv, (void*)&a};
+    s = launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(32 * (NW + 1)), smem, st, args,
+                   "attn_bf16_kernel launch");
+    if (s != SBD_OK) return s;
   }
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "attn_bf16_kernel launch");
+  }
   if (p.splits > 1) {
-    const size_t cs = ((size_t)p.splits + 1) * p.M * sizeof(float);
-    attn_combine_kernel<__nv_bfloat16><<<p.B * p.Hkv, 256, cs, st>>>(
-        a.part_o, a.part_lse, (__nv_bfloat16*)out, p.B, p.k, p.Hq, p.Hkv, p.G, p.M, p.D,
-        p.splits);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_fail(e, "attn_combine_kernel launch");
+    const float* po = a.part_o;
+    const float* pl = a.part_lse;
+    __nv_bfloat16* o = (__nv_bfloat16*)out;
+    int k = p.k, Hq = p.Hq, Hkv = p.Hkv, G = p.G, M = p.M, D = p.D, S = p.splits;
+    void* args[] = {(void*)&po, (void*)&pl, (void*)&o, (void*)&k, (void*)&Hq, (void*)&Hkv,
+                    (void*)&G,  (void*)&M,  (void*)&D, (void*)&S};
+    s = launch_pdl((const void*)attn_combine_kernel<__nv_bfloat16>, dim3(p.M, p.Hkv, p.B),
+                   dim3(128), 0, st, args, "attn_combine_kernel launch");
+    if (s != SBD_OK) return s;
   }
   return SBD_OK;
 }

@@ -1,0 +1,561 @@
+// Block attention on the tcgen05 tensor cores (arXiv 2509.04185, Eq. 5;
+// inference mask of Fig. 3) for bf16 inputs.
+//
+// Same partition as the mma.sync kernel -- one CTA per (KV split, KV head,
+// sequence), the G query heads of a KV head packed with the k block rows
+// into one row tile (row r = i*G + g, padded to 128) -- but both products run
+// on tcgen05 with their accumulators in tensor memory:
+//
+//   S_j = Q K_j^T     A = Q (shared, K-major), B = K tile (shared, K-major),
+//                     M = 128 rows, N = 64 keys, fp32 in TMEM (2 buffers);
+//   O  += P_j V_j     A = P_j (bf16, shared, K-major), B = V tile (shared,
+//                     MN-major: keys are K, head dims N), fp32 O in TMEM.
+//
+// Warp roles: warp 0 streams K/V tiles with TMA (4-stage ring) and copies
+// the k block keys/values as the last tile of the last split; warp 1 owns
+// the tensor memory and one thread issues the MMAs, computing S_{j+1} while
+// the softmax of tile j runs; warps 2-5 are the softmax: thread = row, it
+// reads its 64 scores with tcgen05.ld, applies the mask (cache key < L_b,
+// block key < k) and the scale, and writes P_j = 2^(s - m_ref) as bf16 into
+// shared memory.  The reference max m_ref only moves (and O is rescaled in
+// tensor memory) when the running max exceeds it by more than 2^8, which
+// keeps every P entry <= 256; l and O use the same reference, so the result
+// is exact.  The epilogue normalises O by l and writes the output (one split)
+// or the split partial and its log-sum-exp.
+#include <math.h>
+
+#include "sbd_internal.cuh"
+
+namespace {
+
+using namespace sbd_dev;
+
+constexpr int kTileKeys = 64;
+constexpr int kMaxStages = 6;
+constexpr int kRows = 128;                 // MMA M (packed rows, padded)
+constexpr int kThreads = 192;              // producer, MMA, 4 softmax warps
+constexpr float kRescaleThreshold = 8.f;   // log2 units
+// Cache tiles are prefetched into L2 this many tiles ahead of the ring, so
+// that the ring's loads see L2 rather than HBM latency.
+#ifndef SBD_ATTN_L2_AHEAD
+#define SBD_ATTN_L2_AHEAD 8
+#endif
+
+// ------------------------------------------------------------ tcgen05 PTX
+__device__ __forceinline__ void tc_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tc_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tc_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory descriptor of a 128-byte-swizzled operand: lbo/sbo in bytes.
+// K-major: rows 128 B apart, 8-row groups `sbo` apart (lbo unused).
+// MN-major: 64-element atoms along MN `lbo` apart, 8-row groups along K
+// `sbo` apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
+// kind::f16 instruction descriptor: bf16 A and B, fp32 D; b_mn = B is MN-major.
+__device__ __forceinline__ uint32_t idesc_bf16(int M, int N, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Address of (row, 16-byte chunk c) inside a [rows x 128 B] swizzled tile.
+__device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk) {
+  return base + row * 128 + (((chunk ^ (row & 7)) & 7) << 4);
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+struct TcArgs {
+  const __nv_bfloat16* q;
+  const __nv_bfloat16* kb;
+  const __nv_bfloat16* vb;
+  const int32_t* lens;
+  __nv_bfloat16* out;
+  float* part_o;
+  float* part_lse;
+  int* err;
+  int B, k, Hq, Hkv, G, M, Lmax, splits;
+  float scale_log2;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
+               const __grid_constant__ CUtensorMap tmap_v, const TcArgs a) {
+  constexpr int kSub = D / 64;                    // 128-B column sub-tiles
+  constexpr int kQBytes = kRows * 128;            // one Q (or P) sub-tile: 16 KB
+  constexpr int kKVSub = kTileKeys * 128;         // one K or V sub-tile: 8 KB
+  constexpr int kStageBytes = 2 * kSub * kKVSub;  // K sub-tiles then V sub-tiles
+  constexpr uint32_t kTmemCols = 256;             // S0 | S1 | O
+  constexpr uint32_t kOCol = 2 * kTileKeys;
+  // With D = 128 the K region of a stage (16 KB) is exactly a P tile, and K is
+  // dead once S_j is computed: P_j is written there, and the ring gets the
+  // shared memory separate P buffers would take.
+  constexpr bool kPInK = D == 128;
+  constexpr int kStages = kPInK ? 6 : 5;
+
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t kv_full[kMaxStages], kv_empty[kMaxStages];
+  __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
+  __shared__ __align__(8) uint64_t q_ready, tail_bar;
+  __shared__ uint32_t tmem_base_sh;
+
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t q_s = sbase;                              // kSub x 16 KB
+  const uint32_t p_s = q_s + kSub * kQBytes;               // 2 x 16 KB unless kPInK
+  const uint32_t kv_s = p_s + (kPInK ? 0 : 2 * kQBytes);   // kStages x kStageBytes
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 4);      // one arrival per softmax warp
+      mbar_init(&p_full[i], 4);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(&q_ready, 4);
+    mbar_init(&tail_bar, 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) tc_alloc(&tmem_base_sh, kTmemCols);
+  grid_dependency_wait();
+
+  int len = a.lens[b];
+  if (len < 0 || len > a.Lmax) {
+    if (threadIdx.x == 0 && split == 0 && hkv == 0) record_error(a.err, SBD_DEVERR_CACHE_LEN);
+    len = len < 0 ? 0 : a.Lmax;
+  }
+  const int n_cache_tiles = (len + kTileKeys - 1) / kTileKeys;
+  const int n_tiles = n_cache_tiles + 1;
+  const int t_begin = (int)((long long)split * n_tiles / a.splits);
+  const int t_end = (int)((long long)(split + 1) * n_tiles / a.splits);
+  const int n = t_end - t_begin;
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_sh;
+
+  if (warp == 0) {
+    // ------------------------------------------------ producer warp
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap_k);
+      tma_prefetch_desc(&tmap_v);
+    }
+    auto prefetch = [&](int t) {
+      if (SBD_ATTN_L2_AHEAD > 0 && t < t_end && t < n_cache_tiles) {
+        for (int h = 0; h < kSub; ++h) {
+          tma_prefetch_l2_4d(&tmap_k, 64 * h, hkv, t * kTileKeys, b);
+          tma_prefetch_l2_4d(&tmap_v, 64 * h, hkv, t * kTileKeys, b);
+        }
+      }
+    };
+    if (lane == 0)
+      for (int t = t_begin + kStages; t < t_begin + kStages + SBD_ATTN_L2_AHEAD; ++t) prefetch(t);
+    for (int j = 0; j < n; ++j) {
+      const int t = t_begin + j;
+      const int stage = j % kStages;
+      const uint32_t ph = (j / kStages) & 1;
+      if (!mbar_wait(&kv_empty[stage], ph ^ 1, a.err)) break;
+      const uint32_t ks = kv_s + stage * kStageBytes;
+      const uint32_t vs = ks + kSub * kKVSub;
+      uint8_t* kg = smem_raw + (ks - smem_u32(smem_raw));
+      uint8_t* vg = smem_raw + (vs - smem_u32(smem_raw));
+      if (t < n_cache_tiles) {
+        const int valid = min(kTileKeys, len - t * kTileKeys);
+        const bool tail = valid < kTileKeys;
+        uint64_t* bar = tail ? &tail_bar : &kv_full[stage];
+        if (lane == 0) {
+          prefetch(t + kStages + SBD_ATTN_L2_AHEAD);
+          mbar_arrive_expect_tx(bar, kStageBytes);
+          for (int h = 0; h < kSub; ++h) {
+            tma_load_4d(kg + h * kKVSub, &tmap_k, bar, 64 * h, hkv, t * kTileKeys, b);
+            tma_load_4d(vg + h * kKVSub, &tmap_v, bar, 64 * h, hkv, t * kTileKeys, b);
+          }
+        }
+        if (tail) {
+          // The last cache tile: value rows past the length may hold anything
+          // (NaN); zero them so that zero probabilities stay zero.
+          mbar_wait(&tail_bar, 0, a.err);
+          for (int c = lane; c < (kTileKeys - valid) * kSub * 8; c += 32) {
+            const int row = valid + c / (kSub * 8), h = (c / 8) % kSub, cc = c % 8;
+            st_shared_v4(swz(vs + h * kKVSub, row, cc), make_uint4(0, 0, 0, 0));
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&kv_full[stage]);
+        }
+      } else {
+        // Block keys/values (not cached): rows j < k copied, rows k..63 zero.
+        for (int c = lane; c < kTileKeys * kSub * 8; c += 32) {
+          const int row = c / (kSub * 8), cc = c % (kSub * 8);
+          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+          if (row < a.k) {
+            const size_t off = (((size_t)b * a.k + row) * a.Hkv + hkv) * D + cc * 8;
+            kv = *reinterpret_cast<const uint4*>(a.kb + off);
+            vv = *reinterpret_cast<const uint4*>(a.vb + off);
+          }
+          st_shared_v4(swz(ks + (cc / 8) * kKVSub, row, cc % 8), kv);
+          st_shared_v4(swz(vs + (cc / 8) * kKVSub, row, cc % 8), vv);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&kv_full[stage]);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0 && n > 0) {
+      const uint32_t id_s = idesc_bf16(kRows, kTileKeys, false);
+      const uint32_t id_o = idesc_bf16(kRows, D, true);
+      bool ok = mbar_wait(&q_ready, 0, a.err);
+      tc_fence_after();
+      auto issue_s = [&](int j) {
+        const uint32_t ks = kv_s + (j % kStages) * kStageBytes;
+        const uint32_t d = tmem + (uint32_t)((j & 1) * kTileKeys);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t ad = sw128_desc(q_s + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
+          const uint64_t bd = sw128_desc(ks + (kk / 4) * kKVSub + (kk % 4) * 32, 16, 1024);
+          tc_mma(d, ad, bd, id_s, kk > 0);
+        }
+        tc_commit(&s_full[j & 1]);
+      };
+      auto issue_pv = [&](int j) {
+        const uint32_t ps = kPInK ? kv_s + (j % kStages) * kStageBytes : p_s + (j & 1) * kQBytes;
+        const uint32_t vs = kv_s + (j % kStages) * kStageBytes + kSub * kKVSub;
+#pragma unroll
+        for (int kk = 0; kk < kTileKeys / 16; ++kk) {
+          const uint64_t ad = sw128_desc(ps + kk * 32, 16, 1024);
+          const uint64_t bd = sw128_desc(vs + kk * 16 * 128, kKVSub, 1024);
+          tc_mma(tmem + kOCol, ad, bd, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(&pv_done[j & 1]);
+        tc_commit(&kv_empty[j % kStages]);
+      };
+      // In order: S_{j+1} is issued before waiting for P_j, so the scores of
+      // the next tile are computed while the softmax of this one runs; and
+      // since S_{j+1} is issued after PV_{j-1}, the completion of S_{j+1}
+      // (s_full) implies PV_{j-1} is done, which keeps every later parity
+      // wait on pv_done at most one phase behind.
+      auto wait_issue_s = [&](int j) -> bool {
+        if (!mbar_wait(&kv_full[j % kStages], (j / kStages) & 1, a.err)) return false;
+        if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1, a.err)) return false;
+        tc_fence_after();
+        issue_s(j);
+        return true;
+      };
+      if (ok) ok = wait_issue_s(0);
+      for (int j = 0; j < n && ok; ++j) {
+        if (j + 1 < n && !wait_issue_s(j + 1)) break;
+        if (!mbar_wait(&p_full[j & 1], (j >> 1) & 1, a.err)) break;
+        tc_fence_after();
+        issue_pv(j);
+      }
+    }
+  } else {
+    // ------------------------------------------------ softmax warps
+    const int quad = warp & 3;                  // TMEM lanes 32*quad .. +31
+    const int row = quad * 32 + lane;           // packed row = TMEM lane
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    // Q row -> shared (swizzled, K-major); padding rows are zero.
+    {
+      const __nv_bfloat16* qrow =
+          row < a.M ? a.q + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
+                    : nullptr;
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) {
+        const uint4 v = qrow ? *reinterpret_cast<const uint4*>(qrow + c * 8) : make_uint4(0, 0, 0, 0);
+        st_shared_v4(swz(q_s + (c / 8) * kQBytes, row, c % 8), v);
+      }
+      if (!kPInK && quad * 32 >= a.M) {
+        // rows of these warps are never written: keep their P rows zero
+        for (int c = 0; c < 8; ++c) {
+          st_shared_v4(swz(p_s, row, c), make_uint4(0, 0, 0, 0));
+          st_shared_v4(swz(p_s + kQBytes, row, c), make_uint4(0, 0, 0, 0));
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&q_ready);
+    }
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n && ok; ++j) {
+      const int t = t_begin + j;
+      const int valid = t < n_cache_tiles ? min(kTileKeys, len - t * kTileKeys) : a.k;
+      if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float s[kTileKeys];
+      {
+        uint32_t r0[16], r1[16], r2[16], r3[16];
+        const uint32_t sa = tmem + lane_addr + (uint32_t)((j & 1) * kTileKeys);
+        tc_ld16(sa, r0);
+        tc_ld16(sa + 16, r1);
+        tc_ld16(sa + 32, r2);
+        tc_ld16(sa + 48, r3);
+        tc_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          s[e] = __uint_as_float(r0[e]);
+          s[16 + e] = __uint_as_float(r1[e]);
+          s[32 + e] = __uint_as_float(r2[e]);
+          s[48 + e] = __uint_as_float(r3[e]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[j & 1]);
+      // masked keys only exist in the last cache tile and the block tile
+      if (valid < kTileKeys) {
+#pragma unroll
+        for (int c = 0; c < kTileKeys; ++c)
+          if (c >= valid) s[c] = -INFINITY;
+      }
+      float mx[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = s[e];
+#pragma unroll
+      for (int c = 8; c < kTileKeys; c += 8)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[c + e]);
+      const float mraw = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      const float mt = mraw * a.scale_log2;     // the scale is positive
+      const bool rescale = m_ref != -INFINITY && mt > m_ref + kRescaleThreshold;
+      // The P buffer of this tile is free once PV(j-2) is done; O itself is
+      // only touched (rescaled) after PV(j-1).
+      const int wait_j = rescale ? j - 1 : (kPInK ? -1 : j - 2);
+      if (wait_j >= 0 && !mbar_wait(&pv_done[wait_j & 1], (wait_j >> 1) & 1, a.err)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (m_ref == -INFINITY) {
+        m_ref = mt;
+      } else if (rescale) {
+        const float alpha = exp2f(m_ref - mt);
+        l *= alpha;
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+        }
+        tc_wait_st();
+        m_ref = mt;
+      }
+      // P = 2^(scale * s - m_ref) as bf16 into the tile's P buffer (row =
+      // thread); warps holding only padding rows write zeros.
+      const uint32_t pb =
+          kPInK ? kv_s + (j % kStages) * kStageBytes : p_s + (j & 1) * kQBytes;
+      if (quad * 32 < a.M) {
+        const float nm = -m_ref;
+        float psum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < kTileKeys / 8; ++c) {
+          float p[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            p[e] = exp2f(fmaf(s[c * 8 + e], a.scale_log2, nm));
+            psum[e] += p[e];
+          }
+          st_shared_v4(swz(pb, row, c), make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
+                                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7])));
+        }
+        l += ((psum[0] + psum[1]) + (psum[2] + psum[3])) + ((psum[4] + psum[5]) + (psum[6] + psum[7]));
+      } else if (kPInK) {
+        // the K tile under this P tile is not zero: clear the padding rows
+#pragma unroll
+        for (int c = 0; c < kTileKeys / 8; ++c) st_shared_v4(swz(pb, row, c), make_uint4(0, 0, 0, 0));
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[j & 1]);
+    }
+    grid_dependents_launch();
+    // ------------------------------------------------ epilogue
+    if (ok && n > 0 && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err)) {
+      tc_fence_after();
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const bool mine = row < a.M;
+      if (a.splits == 1) {
+        __nv_bfloat16* dst =
+            mine ? a.out + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
+                 : nullptr;
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+          if (mine) {
+            uint4 w0, w1;
+            w0.x = pack_bf16(__uint_as_float(r[0]) * inv, __uint_as_float(r[1]) * inv);
+            w0.y = pack_bf16(__uint_as_float(r[2]) * inv, __uint_as_float(r[3]) * inv);
+            w0.z = pack_bf16(__uint_as_float(r[4]) * inv, __uint_as_float(r[5]) * inv);
+            w0.w = pack_bf16(__uint_as_float(r[6]) * inv, __uint_as_float(r[7]) * inv);
+            w1.x = pack_bf16(__uint_as_float(r[8]) * inv, __uint_as_float(r[9]) * inv);
+            w1.y = pack_bf16(__uint_as_float(r[10]) * inv, __uint_as_float(r[11]) * inv);
+            w1.z = pack_bf16(__uint_as_float(r[12]) * inv, __uint_as_float(r[13]) * inv);
+            w1.w = pack_bf16(__uint_as_float(r[14]) * inv, __uint_as_float(r[15]) * inv);
+            *reinterpret_cast<uint4*>(dst + c * 16) = w0;
+            *reinterpret_cast<uint4*>(dst + c * 16 + 8) = w1;
+          }
+        }
+      } else {
+        const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
+        float* dst = mine ? a.part_o + prow * D : nullptr;
+#pragma unroll
+        for (int c = 0; c < D / 16; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+          if (mine) {
+#pragma unroll
+            for (int e = 0; e < 16; e += 4)
+              *reinterpret_cast<float4*>(dst + c * 16 + e) =
+                  make_float4(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv,
+                              __uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
+          }
+        }
+        if (mine) a.part_lse[prow] = l > 0.f ? m_ref + log2f(l) : -INFINITY;
+      }
+    } else if (n == 0 && a.splits > 1 && row < a.M) {
+      // an empty split contributes nothing
+      const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
+      for (int d = 0; d < D; ++d) a.part_o[prow * D + d] = 0.f;
+      a.part_lse[prow] = -INFINITY;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tc_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+namespace sbd {
+
+size_t attn_tc_smem_bytes(int D) {
+  const int sub = D / 64;
+  const bool p_in_k = D == 128;
+  const int stages = p_in_k ? 6 : 5;
+  return 1024 + (size_t)sub * kRows * 128 + (p_in_k ? 0 : 2 * kRows * 128) +
+         (size_t)stages * 2 * sub * kTileKeys * 128;
+}
+
+sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
+                          const void* q, const int32_t* lens, const void* kb, const void* vb,
+                          void* out, float* part_o, float* part_lse, cudaStream_t st) {
+  TcArgs a;
+  a.q = (const __nv_bfloat16*)q;
+  a.kb = (const __nv_bfloat16*)kb;
+  a.vb = (const __nv_bfloat16*)vb;
+  a.lens = lens;
+  a.out = (__nv_bfloat16*)out;
+  a.part_o = part_o;
+  a.part_lse = part_lse;
+  a.err = device_error_word();
+  a.B = p.B;
+  a.k = p.k;
+  a.Hq = p.Hq;
+  a.Hkv = p.Hkv;
+  a.G = p.G;
+  a.M = p.M;
+  a.Lmax = p.Lmax;
+  a.splits = p.splits;
+  a.scale_log2 = p.scale_log2;
+  const size_t smem = attn_tc_smem_bytes(p.D);
+  const void* fn = p.D == 128 ? (const void*)attn_tc_kernel<128> : (const void*)attn_tc_kernel<64>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
+  CUtensorMap k_map = tk, v_map = tv;
+  void* args[] = {(void*)&k_map, (void*)&v_map, (void*)&a};
+  return launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(kThreads), smem, st, args,
+                    "attn_tc_kernel launch");
+}
+
+}  // namespace sbd

@@ -10,6 +10,8 @@
 
 namespace {
 
+using namespace sbd_dev;
+
 constexpr int kWarpsPerBlock = 4;
 
 __device__ __forceinline__ bool key_less(float ha, int ia, float hb, int ib) {
@@ -20,6 +22,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock)
 eb_select_kernel(int B, int k, const float* __restrict__ entropy,
                  const int32_t* __restrict__ token, float gamma, uint8_t* __restrict__ masked,
                  int32_t* __restrict__ block_tokens, int32_t* __restrict__ n_unmasked) {
+  grid_dependency_wait();
+  grid_dependents_launch();
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   if (b >= B) return;
@@ -87,11 +91,10 @@ sbd_status eb_launch(int B, int k, const float* entropy, const int32_t* token, f
                      cudaStream_t st) {
   if (B == 0) return SBD_OK;
   const int blocks = (B + kWarpsPerBlock - 1) / kWarpsPerBlock;
-  eb_select_kernel<<<blocks, 32 * kWarpsPerBlock, 0, st>>>(B, k, entropy, token, gamma, masked,
-                                                           block_tokens, n_unmasked);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "eb_select_kernel launch");
-  return SBD_OK;
+  void* args[] = {(void*)&B,      (void*)&k,      (void*)&entropy,      (void*)&token,
+                  (void*)&gamma,  (void*)&masked, (void*)&block_tokens, (void*)&n_unmasked};
+  return launch_pdl((const void*)eb_select_kernel, dim3(blocks), dim3(32 * kWarpsPerBlock), 0, st,
+                    args, "eb_select_kernel launch");
 }
 
 }  // namespace sbd

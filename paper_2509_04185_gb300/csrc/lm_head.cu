@@ -28,9 +28,26 @@ namespace {
 using namespace sbd_dev;
 
 constexpr int kBM = 128;              // vocab rows per tile (MMA M)
-constexpr int kBK = 64;               // hidden columns per stage (one 128-B swizzle atom)
-constexpr int kABytes = kBM * kBK * 2;
+constexpr int kBK = 64;               // hidden columns per TMA box (one 128-B swizzle atom)
+constexpr int kABytes = kBM * kBK * 2;  // one W box
 constexpr int kMaxStages = 16;
+// A pipeline stage holds up to this many consecutive boxes along the hidden
+// dimension (longer contiguous reads of every W row per stage), and the ring
+// gets this many bytes of shared memory.
+#ifndef SBD_HEAD_MAX_BOXES
+#define SBD_HEAD_MAX_BOXES 4
+#endif
+#ifndef SBD_HEAD_RING_BYTES
+#define SBD_HEAD_RING_BYTES (216 * 1024)
+#endif
+// Resident CTAs per SM (the ring budget is shared between them) and whether
+// W is loaded with an L2 evict-first policy.
+#ifndef SBD_HEAD_CTAS_PER_SM
+#define SBD_HEAD_CTAS_PER_SM 1
+#endif
+#ifndef SBD_HEAD_EVICT_FIRST
+#define SBD_HEAD_EVICT_FIRST 1
+#endif
 constexpr int kHeadThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -105,35 +122,55 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
 }
 
 // ------------------------------------------------------------ epilogue math
-// Reduces one logit column over the 32 lanes of a warp (lane = vocab id v).
+__device__ __forceinline__ RowStats shfl_xor_stats(const RowStats& a, int o) {
+  RowStats r;
+  r.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+  r.S = __shfl_xor_sync(0xffffffffu, a.S, o);
+  r.T = __shfl_xor_sync(0xffffffffu, a.T, o);
+  r.best = __shfl_xor_sync(0xffffffffu, a.best, o);
+  r.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
+  return r;
+}
+
+// Statistics of one logit (this lane's vocabulary id v, one column).
+__device__ __forceinline__ RowStats lane_stats(float z, bool valid, float g, float tau, int v) {
+  RowStats r;
+  r.m = valid ? z * kLog2e : -INFINITY;
+  r.S = valid ? 1.f : 0.f;
+  r.T = 0.f;
+  r.best = valid ? fmaf(tau, g, z) : -INFINITY;
+  r.idx = valid ? v : 0x7fffffff;
+  return r;
+}
+
+// Reduces one column over the 32 lanes of a warp; every lane gets the result.
 __device__ __forceinline__ RowStats warp_column_stats(float z, bool valid, float g, float tau,
                                                       int v) {
-  const float y = valid ? z * kLog2e : -INFINITY;
-  const float m = warp_max(y);
-  float e = 0.f, t = 0.f;
-  if (valid && m != -INFINITY) {
-    const float dy = y - m;
-    e = exp2f(dy);
-    t = e * dy;
-  }
-  RowStats r;
-  r.m = m;
-  r.S = warp_sum(e);
-  r.T = warp_sum(t);
-  float best = valid ? fmaf(tau, g, z) : -INFINITY;
-  int idx = valid ? v : 0x7fffffff;
+  RowStats st = lane_stats(z, valid, g, tau, v);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-    if (ob > best || (ob == best && oi < idx)) {
-      best = ob;
-      idx = oi;
+  for (int o = 16; o > 0; o >>= 1) st = rowstats_merge(st, shfl_xor_stats(st, o));
+  return st;
+}
+
+// Reduces 16 columns over the 32 lanes of a warp at once (lane = vocabulary
+// row): at each level a lane keeps half of its columns and merges in the
+// partner lane's copy of them, so 16 + 8 + 4 + 2 + 1 merges replace
+// 16 x 5 full warp reductions.  On return st[0] of lanes 2c and 2c + 1
+// holds column c.
+__device__ __forceinline__ void butterfly16(RowStats (&st)[16], int lane) {
+#pragma unroll
+  for (int lvl = 0; lvl < 4; ++lvl) {
+    const int b = 16 >> lvl;           // lane bit of this level
+    const int half = 8 >> lvl;         // columns kept
+    const bool upper = (lane & b) != 0;
+#pragma unroll
+    for (int i = 0; i < half; ++i) {
+      const RowStats keep = upper ? st[i + half] : st[i];
+      const RowStats send = upper ? st[i] : st[i + half];
+      st[i] = rowstats_merge(keep, shfl_xor_stats(send, b));
     }
   }
-  r.best = best;
-  r.idx = idx;
-  return r;
+  st[0] = rowstats_merge(st[0], shfl_xor_stats(st[0], 1));
 }
 
 struct StatsRef {
@@ -161,12 +198,18 @@ compact_rows_kernel(const uint8_t* __restrict__ hidden, const uint8_t* __restric
                     int BK, int row_bytes, uint8_t* __restrict__ hidden_c,
                     int32_t* __restrict__ row_map, int32_t* __restrict__ n_rows,
                     float* __restrict__ entropy, int32_t* __restrict__ token) {
+  grid_dependency_wait();
   grid_dependents_launch();
   const int row = blockIdx.x;
   const int t = threadIdx.x;
-  const bool mt = t < BK && masked[t] != 0;
-  const int before = __syncthreads_count(mt && t < row);
-  const int total = __syncthreads_count(mt);
+  // masked rows before `row`, and in total (BK <= 2 * blockDim.x)
+  int before = 0, total = 0;
+  for (int base = 0; base < BK; base += blockDim.x) {
+    const int i = base + t;
+    const bool mt = i < BK && masked[i] != 0;
+    before += __syncthreads_count(mt && i < row);
+    total += __syncthreads_count(mt);
+  }
   int dst;
   bool copy = false;
   if (row < BK) {
@@ -199,12 +242,13 @@ struct HeadArgs {
   float4* part_msTb;     // [gridDim.x][rows_alloc]
   int32_t* part_idx;
   int* err;
-  int V, H, rows_alloc, n_tiles, stages;
+  int V, H, rows_alloc, n_tiles, stages, boxes;
+  int n_acc;            // accumulator buffers in tensor memory (2, or 1 above 256 rows)
   uint32_t tmem_cols;
   float tau;
 };
 
-__global__ void __launch_bounds__(kHeadThreads, 1)
+__global__ void __launch_bounds__(kHeadThreads, SBD_HEAD_CTAS_PER_SM)
 head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                const __grid_constant__ CUtensorMap tmap_h, const HeadArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -217,8 +261,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (sbase - smem_u32(smem_raw));
-  const int b_bytes = a.rows_alloc * kBK * 2;
-  const int stage_bytes = kABytes + b_bytes;
+  const int b_box = a.rows_alloc * kBK * 2;            // one hidden-row box
+  const int stage_bytes = a.boxes * (kABytes + b_box);  // [A boxes | B boxes]
   // epilogue scratch after the ring
   uint8_t* ep = gbase + (size_t)a.stages * stage_bytes;
   StatsRef wstats[4];
@@ -236,7 +280,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tmem_full[i], 1);
-      mbar_init(&tmem_empty[i], 128);
+      mbar_init(&tmem_empty[i], 4);     // one arrival per epilogue warp
     }
     fence_mbar_init();
   }
@@ -260,7 +304,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
   const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
-  const int num_kb = a.H / kBK;
+  const int num_kb = a.H / (kBK * a.boxes);
 
   if (R > 0) {
     if (warp == 0) {
@@ -278,9 +322,20 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
               break;
             }
             uint8_t* st = gbase + (size_t)s * stage_bytes;
-            mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
-            tma_load_2d_hint(st, &tmap_w, &full_bar[s], kb * kBK, tile * kBM, policy);
-            tma_load_2d(st + kABytes, &tmap_h, &full_bar[s], kb * kBK, 0);
+            mbar_arrive_expect_tx(&full_bar[s], a.boxes * (kABytes + n_eff * kBK * 2));
+            for (int x = 0; x < a.boxes; ++x) {
+              const int col = (kb * a.boxes + x) * kBK;
+#if SBD_HEAD_EVICT_FIRST
+              tma_load_2d_hint(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM, policy);
+#else
+              (void)policy;
+              tma_load_2d(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM);
+#endif
+              // hidden rows in boxes of 16: only the n_eff rows the MMA reads
+              for (int r0 = 0; r0 < n_eff; r0 += 16)
+                tma_load_2d(st + a.boxes * kABytes + x * b_box + r0 * 128, &tmap_h, &full_bar[s],
+                            col, r0);
+            }
           }
         }
         // copies still in flight must land before the CTA exits
@@ -290,12 +345,15 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     } else if (warp == 1) {
       // ------------------------------------------------ MMA issuer
       if (lane == 0) {
-        const uint32_t idesc = idesc_bf16_f32(kBM, n_eff);
+        // N is split into MMAs of at most 256 columns
+        const int n_hi = n_eff > 256 ? n_eff - 256 : 0;
+        const uint32_t idesc_lo = idesc_bf16_f32(kBM, n_eff > 256 ? 256 : n_eff);
+        const uint32_t idesc_hi = idesc_bf16_f32(kBM, n_hi > 0 ? n_hi : 16);
         int it = 0, local = 0;
         bool ok = true;
         for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += gridDim.x, ++local) {
-          const int acc = local & 1;
-          const uint32_t use = (uint32_t)(local >> 1);
+          const int acc = a.n_acc == 2 ? (local & 1) : 0;
+          const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
           if (!mbar_wait(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)(acc * a.rows_alloc);
@@ -308,11 +366,18 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
             }
             tc_fence_after();
             const uint32_t st = sbase + (uint32_t)(s * stage_bytes);
-            const uint64_t adesc = sw128_kmajor_desc(st);
-            const uint64_t bdesc = sw128_kmajor_desc(st + kABytes);
+            for (int x = 0; x < a.boxes; ++x) {
+              const uint64_t adesc = sw128_kmajor_desc(st + x * kABytes);
+              const uint64_t bdesc = sw128_kmajor_desc(st + a.boxes * kABytes + x * b_box);
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-              tc_mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
+              for (int kk = 0; kk < kBK / 16; ++kk) {
+                const uint32_t accum = (kb | x | kk) != 0;
+                tc_mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc_lo, accum);
+                if (n_hi > 0)   // rows 256.. of B: 256 x 128 B further on, 256 columns on
+                  tc_mma_bf16(d_tmem + 256, adesc + 2 * kk, bdesc + (256 * 128 >> 4) + 2 * kk,
+                              idesc_hi, accum);
+              }
+            }
             tc_commit(&empty_bar[s]);
           }
           if (ok) tc_commit(&tmem_full[acc]);
@@ -325,16 +390,22 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const bool noisy = a.tau != 0.f && a.gumbel != nullptr;
       int local = 0;
       for (int tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++local) {
-        const int acc = local & 1;
-        const uint32_t use = (uint32_t)(local >> 1);
+        const int acc = a.n_acc == 2 ? (local & 1) : 0;
+        const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
         const int v = tile * kBM + quad * 32 + lane;
         const bool valid = v < a.V;
+        // Gumbel noise of the next 16 columns is loaded while the current
+        // ones are reduced.
+        float g[16], g_next[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          g_next[j] = (noisy && valid && j < R) ? __ldg(a.gumbel + (size_t)rmap[j] * a.V + v) : 0.f;
         for (int c0 = 0; c0 < R; c0 += 16) {
-          float g[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            g[j] = 0.f;
-            if (noisy && valid && c0 + j < R) g[j] = __ldg(a.gumbel + (size_t)rmap[c0 + j] * a.V + v);
+            g[j] = g_next[j];
+            const int cn = c0 + 16 + j;
+            g_next[j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
           }
           if (c0 == 0) {
             if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
@@ -345,21 +416,17 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                                (uint32_t)(acc * a.rows_alloc + c0),
                            r);
           tc_wait_ld();
-          RowStats mine = rowstats_empty();
+          RowStats st[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            if (c0 + j < R) {
-              const RowStats cs = warp_column_stats(__uint_as_float(r[j]), valid, g[j], a.tau, v);
-              if (lane == j) mine = cs;
-            }
-          }
-          if (lane < 16 && c0 + lane < R) {
-            const int col = c0 + lane;
-            store_stats(wstats[ew], col, rowstats_merge(load_stats(wstats[ew], col), mine));
-          }
+          for (int j = 0; j < 16; ++j) st[j] = lane_stats(__uint_as_float(r[j]), valid, g[j], a.tau, v);
+          butterfly16(st, lane);
+          const int col = c0 + ((lane >> 1) & 15);
+          if ((lane & 1) == 0 && col < R)
+            store_stats(wstats[ew], col, rowstats_merge(load_stats(wstats[ew], col), st[0]));
         }
         tc_fence_before();
-        mbar_arrive(&tmem_empty[acc]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tmem_empty[acc]);
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
       const int te = threadIdx.x - 64;
@@ -506,17 +573,33 @@ HeadWs head_ws_layout(const sbd::HeadPlan& p, void* base) {
   return w;
 }
 
-int head_stages(int rows_alloc) {
-  const int stage_bytes = kABytes + rows_alloc * kBK * 2;
+int head_ring_budget(int rows_alloc) {
   const int ep_bytes = 4 * rows_alloc * (16 + 4) + rows_alloc * 4;
-  const int budget = 220 * 1024 - 1024 - ep_bytes;
-  int s = budget / stage_bytes;
+  const int per_cta = (224 * 1024) / SBD_HEAD_CTAS_PER_SM - 1024 - 1024;
+  int budget = SBD_HEAD_RING_BYTES / SBD_HEAD_CTAS_PER_SM;
+  if (budget > per_cta - ep_bytes) budget = per_cta - ep_bytes;
+  return budget;
+}
+
+// Boxes per stage: the largest count <= SBD_HEAD_MAX_BOXES that divides the
+// hidden size into whole stages and still leaves at least 3 stages.
+int head_boxes(int H, int rows_alloc) {
+  int nb = SBD_HEAD_MAX_BOXES;
+  while (nb > 1 && ((H / kBK) % nb != 0 ||
+                    head_ring_budget(rows_alloc) / (nb * (kABytes + rows_alloc * kBK * 2)) < 3))
+    nb >>= 1;
+  return nb;
+}
+
+int head_stages(int rows_alloc, int boxes) {
+  const int stage_bytes = boxes * (kABytes + rows_alloc * kBK * 2);
+  int s = head_ring_budget(rows_alloc) / stage_bytes;
   if (s > kMaxStages) s = kMaxStages;
   return s;
 }
 
-size_t head_smem_bytes(int rows_alloc, int stages) {
-  const size_t stage_bytes = kABytes + (size_t)rows_alloc * kBK * 2;
+size_t head_smem_bytes(int rows_alloc, int stages, int boxes) {
+  const size_t stage_bytes = (size_t)boxes * (kABytes + (size_t)rows_alloc * kBK * 2);
   return 1024 + stages * stage_bytes + (size_t)4 * rows_alloc * (16 + 4) + rows_alloc * 4;
 }
 
@@ -535,8 +618,8 @@ HeadPlan head_plan(const sbd_head_desc& d) {
   p.rows_alloc = bk <= 16 ? 16 : ((bk + 15) / 16) * 16;
   const int n_tiles = (d.vocab + kBM - 1) / kBM;
   if (p.bf16) {
-    const int sms = num_sms();
-    p.n_ctas = n_tiles < sms ? n_tiles : sms;
+    const int slots = num_sms() * SBD_HEAD_CTAS_PER_SM;
+    p.n_ctas = n_tiles < slots ? n_tiles : slots;
   } else {
     p.n_ctas = n_tiles;
   }
@@ -545,23 +628,6 @@ HeadPlan head_plan(const sbd_head_desc& d) {
 
 size_t head_workspace_bytes(const HeadPlan& p) { return head_ws_layout(p, nullptr).bytes; }
 
-static sbd_status launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
-                             void** args) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelExC(&cfg, fn, args);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernelExC");
-  return SBD_OK;
-}
-
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
                        int32_t* token, void* ws, cudaStream_t st) {
@@ -569,14 +635,21 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
   if (BK == 0) return SBD_OK;
   HeadWs W = head_ws_layout(p, ws);
   const int elem = p.bf16 ? 2 : 4;
-  compact_rows_kernel<<<p.rows_alloc, 256, 0, st>>>((const uint8_t*)hidden, masked, BK,
-                                                    p.H * elem, W.hidden_c, W.row_map, W.n_rows,
-                                                    entropy, token);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "compact_rows_kernel launch");
-
-  int* err = device_error_word();
   sbd_status s;
+  {
+    const uint8_t* hid = (const uint8_t*)hidden;
+    int bk = BK, rb = p.H * elem;
+    uint8_t* hc = W.hidden_c;
+    int32_t* rm = W.row_map;
+    int32_t* nr = W.n_rows;
+    void* args[] = {(void*)&hid, (void*)&masked, (void*)&bk, (void*)&rb, (void*)&hc,
+                    (void*)&rm,  (void*)&nr,     (void*)&entropy, (void*)&token};
+    s = launch_pdl((const void*)compact_rows_kernel, dim3(p.rows_alloc), dim3(256), 0, st, args,
+                   "compact_rows_kernel launch");
+    if (s != SBD_OK) return s;
+  }
+  cudaError_t e;
+  int* err = device_error_word();
   if (p.bf16) {
     CUtensorMap tw, th;
     {
@@ -590,7 +663,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     {
       const uint64_t dims[2] = {(uint64_t)p.H, (uint64_t)p.rows_alloc};
       const uint64_t strides[1] = {(uint64_t)p.H * 2};
-      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)p.rows_alloc};
+      const uint32_t box[2] = {(uint32_t)kBK, 16u};
       s = encode_tensor_map(&th, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)W.hidden_c, dims,
                             strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
       if (s != SBD_OK) return s;
@@ -606,18 +679,20 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.H = p.H;
     a.rows_alloc = p.rows_alloc;
     a.n_tiles = (p.V + kBM - 1) / kBM;
-    a.stages = head_stages(p.rows_alloc);
+    a.boxes = head_boxes(p.H, p.rows_alloc);
+    a.stages = head_stages(p.rows_alloc, a.boxes);
+    a.n_acc = 2 * p.rows_alloc <= 512 ? 2 : 1;
     uint32_t cols = 32;
-    while (cols < (uint32_t)(2 * p.rows_alloc)) cols <<= 1;
+    while (cols < (uint32_t)(a.n_acc * p.rows_alloc)) cols <<= 1;
     a.tmem_cols = cols;
     a.tau = tau;
-    const size_t smem = head_smem_bytes(p.rows_alloc, a.stages);
+    const size_t smem = head_smem_bytes(p.rows_alloc, a.stages, a.boxes);
     e = cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
     void* args[] = {(void*)&tw, (void*)&th, (void*)&a};
     s = launch_pdl((const void*)head_tc_kernel, dim3(p.n_ctas), dim3(kHeadThreads), smem, st,
-                   args);
+                   args, "head_tc_kernel launch");
     if (s != SBD_OK) return s;
   } else {
     const float* hc = (const float*)W.hidden_c;
@@ -630,7 +705,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     void* args[] = {(void*)&hc, (void*)&wf, (void*)&gumbel, (void*)&rm, (void*)&nr,
                     (void*)&tau, (void*)&V,  (void*)&H,      (void*)&ra, (void*)&pm,
                     (void*)&pi};
-    s = launch_pdl((const void*)head_f32_kernel, dim3(p.n_ctas), dim3(128), 0, st, args);
+    s = launch_pdl((const void*)head_f32_kernel, dim3(p.n_ctas), dim3(128), 0, st, args,
+                   "head_f32_kernel launch");
     if (s != SBD_OK) return s;
   }
   {
@@ -642,7 +718,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     void* args[] = {(void*)&pm, (void*)&pi, (void*)&np, (void*)&ra,
                     (void*)&rm, (void*)&nr, (void*)&entropy, (void*)&token};
     s = launch_pdl((const void*)head_combine_kernel, dim3((p.rows_alloc + 3) / 4), dim3(128), 0,
-                   st, args);
+                   st, args, "head_combine_kernel launch");
     if (s != SBD_OK) return s;
   }
   return SBD_OK;

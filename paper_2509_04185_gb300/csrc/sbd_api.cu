@@ -104,6 +104,23 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
   return SBD_OK;
 }
 
+sbd_status launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                      void** args, const char* what) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelExC(&cfg, fn, args);
+  if (e != cudaSuccess) return cuda_fail(e, what);
+  return SBD_OK;
+}
+
 }  // namespace sbd
 
 using sbd::aligned16;
@@ -149,8 +166,8 @@ sbd_status check_head_desc(const sbd_head_desc* d) {
                 d->batch, d->block_k, d->hidden, d->vocab);
   if (d->dtype != SBD_DTYPE_F32 && d->dtype != SBD_DTYPE_BF16)
     return fail(SBD_ERR_INVALID_ARG, "unknown dtype %d", d->dtype);
-  if ((long long)d->batch * d->block_k > 256)
-    return fail(SBD_ERR_UNSUPPORTED, "batch * block_k = %lld > 256",
+  if ((long long)d->batch * d->block_k > 512)
+    return fail(SBD_ERR_UNSUPPORTED, "batch * block_k = %lld > 512",
                 (long long)d->batch * d->block_k);
   if (d->dtype == SBD_DTYPE_BF16 && d->hidden % 64 != 0)
     return fail(SBD_ERR_UNSUPPORTED, "hidden %d is not a multiple of 64", d->hidden);

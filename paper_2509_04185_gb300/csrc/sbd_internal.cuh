@@ -27,7 +27,7 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
 // Kernel launchers (each in the .cu file of its kernel).  Arguments were
 // validated by the API layer.
 struct AttnPlan {
-  int B, k, Hq, Hkv, G, D, Lmax, M, splits;
+  int B, k, Hq, Hkv, G, D, Lmax, M, splits, stages, MT, KG;
   float scale_log2;   // softmax scale * log2(e)
   bool bf16;
 };
@@ -36,6 +36,11 @@ AttnPlan attn_plan(const sbd_attn_desc& d);
 sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const void* vc,
                        const int32_t* lens, const void* kb, const void* vb, void* out,
                        void* ws, cudaStream_t st);
+
+size_t attn_tc_smem_bytes(int D);
+sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
+                          const void* q, const int32_t* lens, const void* kb, const void* vb,
+                          void* out, float* part_o, float* part_lse, cudaStream_t st);
 
 struct HeadPlan {
   int B, k, H, V, rows_alloc, n_ctas;
@@ -52,6 +57,12 @@ sbd_status eb_launch(int B, int k, const float* entropy, const int32_t* token, f
                      cudaStream_t st);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Launch with programmatic dependent launch allowed: the kernel may be
+// scheduled while its predecessor on the stream finishes; every library
+// kernel calls griddepcontrol.wait before it touches global memory.
+sbd_status launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                      void** args, const char* what);
 
 }  // namespace sbd
 
@@ -102,14 +113,27 @@ __device__ __forceinline__ bool mbar_test_parity(uint64_t* bar, uint32_t parity)
       : "memory");
   return ok != 0;
 }
+// Non-blocking test of the same condition (for polling several barriers).
+__device__ __forceinline__ bool mbar_poll_parity(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 // Waits until the phase with the given parity has completed, for at most
 // kWaitLimitNs.  Returns false (and records SBD_DEVERR_TIMEOUT) on time-out.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
   if (mbar_test_parity(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
-  while (true) {
+  for (uint32_t n = 1;; ++n) {
     if (mbar_test_parity(bar, parity)) return true;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    // the clock is read every 64 polls only
+    if ((n & 63u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
       record_error(err, SBD_DEVERR_TIMEOUT);
       return false;
     }
@@ -150,6 +174,20 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2),
       "r"(c3)
       : "memory");
+}
+// Prefetch of a tensor tile into L2 (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int c0, int c1) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* map, int c0, int c1, int c2,
+                                                   int c3) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
 }
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t p;

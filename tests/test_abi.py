@@ -90,7 +90,7 @@ def test_attention_rejects_null_and_misaligned(sbd):
 
 def test_head_rejects_bad_arguments(sbd):
     a = 1 << 20
-    d = sbd.HeadDesc(16, 17, 4096, 128256, sbd.SBD_DTYPE_BF16)      # 272 rows > 256
+    d = sbd.HeadDesc(32, 17, 4096, 128256, sbd.SBD_DTYPE_BF16)      # 544 rows > 512
     assert sbd.lib.sbd_head_entropy_sample(ctypes.byref(d), a, a, a, a, 1.0, a, a, a, 1 << 30,
                                            None) == sbd.SBD_ERR_UNSUPPORTED
     d = sbd.HeadDesc(1, 16, 4000, 128256, sbd.SBD_DTYPE_BF16)       # H % 64 != 0

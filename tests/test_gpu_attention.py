@@ -108,3 +108,25 @@ def test_sweep_layer_k32(sbd):
     """One layer of the 32-layer sweep at its largest block (k = 32: 128
     packed rows per KV head), batch 16, cache 8192."""
     _run_and_compare(sbd, gen.sweep_workload(32), seed=0)
+
+
+@pytest.mark.parametrize("k,L,splits", [(8, 8192, 0), (8, 8192, 13), (16, 4096, 0), (32, 2048, 3),
+                                        (4, 4096, 0), (12, 1000, 7)])
+def test_repeated_calls_leave_no_device_error(sbd, k, L, splits):
+    """Back-to-back launches (as in a decode loop) of the same call: every
+    bounded wait inside the kernels must succeed, and the result must not
+    change between repetitions."""
+    import torch
+    w = gen.shrink(BF16, batch=16, block_k=k, cache_len=L)
+    d = gen.attention_inputs(w, seed=3, poison_tail=False)
+    t = {x: to_dev(d[x], "bf16") for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    lens = torch.from_numpy(d["cache_len"]).cuda()
+    out0 = sbd.sbd_block_attention(t["q"], t["k_cache"], t["v_cache"], lens, t["k_blk"], t["v_blk"],
+                                   num_splits=splits)
+    ref = out0.clone()
+    for _ in range(30):
+        sbd.sbd_block_attention(t["q"], t["k_cache"], t["v_cache"], lens, t["k_blk"], t["v_blk"],
+                                out0, num_splits=splits)
+    torch.cuda.synchronize()
+    assert sbd.sbd_device_error() == 0
+    assert torch.equal(out0, ref)
