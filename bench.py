@@ -215,7 +215,8 @@ def run_ours(args):
                        dtype=torch.uint8, device=dev)
     ws_h = torch.empty(max(1, sbd.lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(hd))),
                        dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream(dev)
+    # a dedicated stream: the step is captured into a CUDA graph on it
+    stream = torch.cuda.Stream(dev)
     gamma, tau = args.gamma, args.tau
 
     attn_call = sbd.prepare_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"],
@@ -225,19 +226,20 @@ def run_ours(args):
     eb_call = sbd.prepare_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
 
     def step(ev=None):
-        masked.copy_(masked0, non_blocking=True)
-        bt.copy_(bt0, non_blocking=True)
-        if ev is not None:
-            ev[0].record(stream)
-        attn_call()
-        if ev is not None:
-            ev[1].record(stream)
-        head_call()
-        if ev is not None:
-            ev[2].record(stream)
-        eb_call()
-        if ev is not None:
-            ev[3].record(stream)
+        with torch.cuda.stream(stream):
+            masked.copy_(masked0, non_blocking=True)
+            bt.copy_(bt0, non_blocking=True)
+            if ev is not None:
+                ev[0].record(stream)
+            attn_call()
+            if ev is not None:
+                ev[1].record(stream)
+            head_call()
+            if ev is not None:
+                ev[2].record(stream)
+            eb_call()
+            if ev is not None:
+                ev[3].record(stream)
 
     sampler = ClockSampler(local_rank) if rank == 0 else None
     if sampler:
@@ -248,8 +250,23 @@ def run_ours(args):
     if sbd.sbd_device_error() != 0:
         raise RuntimeError("device error word set during warm-up")
 
+    # The whole step (state restore + three library calls, 6-7 kernels with
+    # programmatic dependent launch between them) captured once as a graph.
+    graph = None
+    if not args.no_graph:
+        try:
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                step()
+            for _ in range(3):
+                with torch.cuda.stream(stream):
+                    graph.replay()
+            torch.cuda.synchronize(dev)
+        except Exception as ex:  # capture unsupported here: time the eager step
+            print(f"graph capture failed ({ex}); timing eager steps", file=sys.stderr)
+            graph = None
+
     # ---- timed region: K steps, events on the launching stream
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     if world > 1:
@@ -258,8 +275,12 @@ def run_ours(args):
     if sampler:
         sampler.mark("timed_start")
     start.record(stream)
-    for i in range(args.steps):
-        step(evs[i])
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            if graph is not None:
+                graph.replay()
+            else:
+                step()
     end.record(stream)
     torch.cuda.synchronize(dev)
     if sampler:
@@ -270,12 +291,20 @@ def run_ours(args):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         torch.distributed.barrier()
         total_ms = float(t.item())
-    attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
-    head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
-    eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
     n_accepted = int(n_un.sum().item())
     if sbd.sbd_device_error() != 0:
         raise RuntimeError("device error word set during the timed region")
+
+    # ---- per-call durations (eager steps, events between the calls on the
+    # launching stream): the roofline of the dominant kernel
+    n_ev = max(1, min(args.steps, 500))
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_ev)]
+    for i in range(n_ev):
+        step(evs[i])
+    torch.cuda.synchronize(dev)
+    attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
 
     # ---- end to end through host buffers (pinned), copies inside the region
     e2e = None
@@ -294,19 +323,20 @@ def run_ours(args):
         n_e2e = max(1, min(args.steps, 200))
 
         def e2e_step():
-            for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
-                T[k].copy_(host[k], non_blocking=True)
-            masked.copy_(host["masked"], non_blocking=True)
-            bt.copy_(host["block_tokens"], non_blocking=True)
-            attn_call()
-            head_call()
-            eb_call()
-            res["out"].copy_(out, non_blocking=True)
-            res["ent"].copy_(ent, non_blocking=True)
-            res["tok"].copy_(tok, non_blocking=True)
-            res["masked"].copy_(masked, non_blocking=True)
-            res["bt"].copy_(bt, non_blocking=True)
-            res["n_un"].copy_(n_un, non_blocking=True)
+            with torch.cuda.stream(stream):
+                for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
+                    T[k].copy_(host[k], non_blocking=True)
+                masked.copy_(host["masked"], non_blocking=True)
+                bt.copy_(host["block_tokens"], non_blocking=True)
+                attn_call()
+                head_call()
+                eb_call()
+                res["out"].copy_(out, non_blocking=True)
+                res["ent"].copy_(ent, non_blocking=True)
+                res["tok"].copy_(tok, non_blocking=True)
+                res["masked"].copy_(masked, non_blocking=True)
+                res["bt"].copy_(bt, non_blocking=True)
+                res["n_un"].copy_(n_un, non_blocking=True)
 
         for _ in range(3):
             e2e_step()
@@ -676,6 +706,7 @@ def main():
     ap.add_argument("--tau", type=float, default=1.0)
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--no-graph", action="store_true", help="time eager launches, no CUDA graph")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

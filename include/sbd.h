@@ -146,7 +146,7 @@ sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden
  *     host threads -- race on it: serialise them (one stream, or events).
  *   - Allocates nothing: no cudaMalloc/cudaFree or allocating library call.
  * ---------------------------------------------------------------------- */
-#define SBD_HEAD_NOALLOC_MAX_SCRATCH (4u << 20) /* 4 MiB */
+#define SBD_HEAD_NOALLOC_MAX_SCRATCH (8u << 20) /* 8 MiB */
 
 sbd_status sbd_head_entropy_sample_noalloc(const sbd_head_desc* desc, const void* hidden,
                                            const void* w, const uint8_t* masked,

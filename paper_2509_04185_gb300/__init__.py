@@ -32,7 +32,7 @@ SBD_DTYPE_BF16 = 1
 SBD_DEVERR_CACHE_LEN = 1
 SBD_DEVERR_TIMEOUT = 2
 SBD_DEVERR_ROWS = 4
-SBD_HEAD_NOALLOC_MAX_SCRATCH = 4 << 20
+SBD_HEAD_NOALLOC_MAX_SCRATCH = 8 << 20
 
 # Every symbol include/sbd.h declares.
 EXPORTS = (

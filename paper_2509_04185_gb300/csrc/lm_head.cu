@@ -242,7 +242,8 @@ struct HeadArgs {
   float4* part_msTb;     // [gridDim.x][rows_alloc]
   int32_t* part_idx;
   int* err;
-  int V, H, rows_alloc, n_tiles, stages, boxes;
+  int V, H, rows_alloc, n_tiles;
+  int ring_bytes;       // shared memory of the TMA ring (shaped in the kernel)
   int n_acc;            // accumulator buffers in tensor memory (2, or 1 above 256 rows)
   uint32_t tmem_cols;
   float tau;
@@ -261,10 +262,11 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (sbase - smem_u32(smem_raw));
-  const int b_box = a.rows_alloc * kBK * 2;            // one hidden-row box
-  const int stage_bytes = a.boxes * (kABytes + b_box);  // [A boxes | B boxes]
-  // epilogue scratch after the ring
-  uint8_t* ep = gbase + (size_t)a.stages * stage_bytes;
+  // epilogue scratch first, then the ring
+  uint8_t* ep = gbase;
+  const int ep_bytes = (4 * a.rows_alloc * (16 + 4) + a.rows_alloc * 4 + 1023) & ~1023;
+  uint8_t* ring = gbase + ep_bytes;
+  const uint32_t rbase = sbase + ep_bytes;
   StatsRef wstats[4];
   for (int w = 0; w < 4; ++w) {
     wstats[w].msTb = reinterpret_cast<float4*>(ep) + w * a.rows_alloc;
@@ -273,8 +275,27 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   }
   int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * a.rows_alloc * (sizeof(float4) + 4));
 
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_h);
+  }
+  if (warp == 1) tc_alloc(&tmem_base_sh, a.tmem_cols);
+  // Everything below reads what the compaction kernel wrote.
+  grid_dependency_wait();
+  const int R = *a.n_rows;
+  const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
+  // Ring shape from the actual row count: a stage holds `boxes` 64-column
+  // boxes of W (16 KB each) and of the n_eff hidden rows; as many boxes as
+  // still leave 3 stages, then as many stages as fit.
+  const int b_box = n_eff * kBK * 2;
+  int boxes = SBD_HEAD_MAX_BOXES;
+  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || a.ring_bytes / (boxes * (kABytes + b_box)) < 3))
+    boxes >>= 1;
+  const int stage_bytes = boxes * (kABytes + b_box);     // [A boxes | B boxes]
+  int stages = a.ring_bytes / stage_bytes;
+  if (stages > kMaxStages) stages = kMaxStages;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < a.stages; ++s) {
+    for (int s = 0; s < stages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
@@ -284,14 +305,6 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     }
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmap_w);
-    tma_prefetch_desc(&tmap_h);
-  }
-  if (warp == 1) tc_alloc(&tmem_base_sh, a.tmem_cols);
-  // Everything below reads what the compaction kernel wrote.
-  grid_dependency_wait();
-  const int R = *a.n_rows;
   if (warp >= 2) {
     const int te = threadIdx.x - 64;
     for (int i = te; i < a.rows_alloc; i += 128) {
@@ -303,8 +316,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
-  const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
-  const int num_kb = a.H / (kBK * a.boxes);
+  const int num_kb = a.H / (kBK * boxes);
 
   if (R > 0) {
     if (warp == 0) {
@@ -313,18 +325,18 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint64_t policy = l2_policy_evict_first();
         int it = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += gridDim.x) {
+        for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x) {
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % a.stages;
-            const uint32_t ph = (it / a.stages) & 1;
+            const int s = it % stages;
+            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&empty_bar[s], ph ^ 1, a.err)) {
               ok = false;
               break;
             }
-            uint8_t* st = gbase + (size_t)s * stage_bytes;
-            mbar_arrive_expect_tx(&full_bar[s], a.boxes * (kABytes + n_eff * kBK * 2));
-            for (int x = 0; x < a.boxes; ++x) {
-              const int col = (kb * a.boxes + x) * kBK;
+            uint8_t* st = ring + (size_t)s * stage_bytes;
+            mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+            for (int x = 0; x < boxes; ++x) {
+              const int col = (kb * boxes + x) * kBK;
 #if SBD_HEAD_EVICT_FIRST
               tma_load_2d_hint(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM, policy);
 #else
@@ -333,14 +345,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 #endif
               // hidden rows in boxes of 16: only the n_eff rows the MMA reads
               for (int r0 = 0; r0 < n_eff; r0 += 16)
-                tma_load_2d(st + a.boxes * kABytes + x * b_box + r0 * 128, &tmap_h, &full_bar[s],
+                tma_load_2d(st + boxes * kABytes + x * b_box + r0 * 128, &tmap_h, &full_bar[s],
                             col, r0);
             }
           }
         }
         // copies still in flight must land before the CTA exits
-        for (int q = it - a.stages > 0 ? it - a.stages : 0; q < it; ++q)
-          mbar_wait(&full_bar[q % a.stages], (q / a.stages) & 1, a.err);
+        for (int q = it - stages > 0 ? it - stages : 0; q < it; ++q)
+          mbar_wait(&full_bar[q % stages], (q / stages) & 1, a.err);
       }
     } else if (warp == 1) {
       // ------------------------------------------------ MMA issuer
@@ -351,27 +363,27 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint32_t idesc_hi = idesc_bf16_f32(kBM, n_hi > 0 ? n_hi : 16);
         int it = 0, local = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += gridDim.x, ++local) {
+        for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x, ++local) {
           const int acc = a.n_acc == 2 ? (local & 1) : 0;
           const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
           if (!mbar_wait(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)(acc * a.rows_alloc);
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % a.stages;
-            const uint32_t ph = (it / a.stages) & 1;
+            const int s = it % stages;
+            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&full_bar[s], ph, a.err)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t st = sbase + (uint32_t)(s * stage_bytes);
-            for (int x = 0; x < a.boxes; ++x) {
+            const uint32_t st = rbase + (uint32_t)(s * stage_bytes);
+            for (int x = 0; x < boxes; ++x) {
               const uint64_t adesc = sw128_kmajor_desc(st + x * kABytes);
-              const uint64_t bdesc = sw128_kmajor_desc(st + a.boxes * kABytes + x * b_box);
+              const uint64_t bdesc = sw128_kmajor_desc(st + boxes * kABytes + x * b_box);
 #pragma unroll
               for (int kk = 0; kk < kBK / 16; ++kk) {
-                const uint32_t accum = (kb | x | kk) != 0;
+                const uint32_t accum = (kb != 0 || x != 0 || kk != 0);
                 tc_mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc_lo, accum);
                 if (n_hi > 0)   // rows 256.. of B: 256 x 128 B further on, 256 columns on
                   tc_mma_bf16(d_tmem + 256, adesc + 2 * kk, bdesc + (256 * 128 >> 4) + 2 * kk,
@@ -388,18 +400,22 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const int ew = warp - 2;                 // 0..3
       const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
       const bool noisy = a.tau != 0.f && a.gumbel != nullptr;
+      const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
       for (int tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++local) {
         const int acc = a.n_acc == 2 ? (local & 1) : 0;
         const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
         const int v = tile * kBM + quad * 32 + lane;
         const bool valid = v < a.V;
-        // Gumbel noise of the next 16 columns is loaded while the current
-        // ones are reduced.
+        const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)(acc * a.rows_alloc);
+        // Gumbel noise of the first 16 columns is loaded while the MMAs run,
+        // that of the next 16 while the current ones are reduced.
         float g[16], g_next[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
           g_next[j] = (noisy && valid && j < R) ? __ldg(a.gumbel + (size_t)rmap[j] * a.V + v) : 0.f;
+        if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
+        tc_fence_after();
         for (int c0 = 0; c0 < R; c0 += 16) {
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -407,18 +423,15 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
             const int cn = c0 + 16 + j;
             g_next[j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
           }
-          if (c0 == 0) {
-            if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
-            tc_fence_after();
-          }
           uint32_t r[16];
-          tc_ld_32x32b_x16(tmem_base + ((uint32_t)(quad * 32) << 16) +
-                               (uint32_t)(acc * a.rows_alloc + c0),
-                           r);
+          tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
           tc_wait_ld();
+          float z[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
           RowStats st[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) st[j] = lane_stats(__uint_as_float(r[j]), valid, g[j], a.tau, v);
+          for (int j = 0; j < 16; ++j) st[j] = lane_stats(z[j], valid, g[j], a.tau, v);
           butterfly16(st, lane);
           const int col = c0 + ((lane >> 1) & 15);
           if ((lane & 1) == 0 && col < R)
@@ -573,34 +586,21 @@ HeadWs head_ws_layout(const sbd::HeadPlan& p, void* base) {
   return w;
 }
 
-int head_ring_budget(int rows_alloc) {
-  const int ep_bytes = 4 * rows_alloc * (16 + 4) + rows_alloc * 4;
+int head_ep_bytes(int rows_alloc) {
+  return (4 * rows_alloc * (16 + 4) + rows_alloc * 4 + 1023) & ~1023;
+}
+
+// Shared memory of the ring: SBD_HEAD_RING_BYTES per SM, within what a CTA
+// can have next to the epilogue scratch.
+int head_ring_bytes(int rows_alloc) {
   const int per_cta = (224 * 1024) / SBD_HEAD_CTAS_PER_SM - 1024 - 1024;
   int budget = SBD_HEAD_RING_BYTES / SBD_HEAD_CTAS_PER_SM;
-  if (budget > per_cta - ep_bytes) budget = per_cta - ep_bytes;
+  if (budget > per_cta - head_ep_bytes(rows_alloc)) budget = per_cta - head_ep_bytes(rows_alloc);
   return budget;
 }
 
-// Boxes per stage: the largest count <= SBD_HEAD_MAX_BOXES that divides the
-// hidden size into whole stages and still leaves at least 3 stages.
-int head_boxes(int H, int rows_alloc) {
-  int nb = SBD_HEAD_MAX_BOXES;
-  while (nb > 1 && ((H / kBK) % nb != 0 ||
-                    head_ring_budget(rows_alloc) / (nb * (kABytes + rows_alloc * kBK * 2)) < 3))
-    nb >>= 1;
-  return nb;
-}
-
-int head_stages(int rows_alloc, int boxes) {
-  const int stage_bytes = boxes * (kABytes + rows_alloc * kBK * 2);
-  int s = head_ring_budget(rows_alloc) / stage_bytes;
-  if (s > kMaxStages) s = kMaxStages;
-  return s;
-}
-
-size_t head_smem_bytes(int rows_alloc, int stages, int boxes) {
-  const size_t stage_bytes = (size_t)boxes * (kABytes + (size_t)rows_alloc * kBK * 2);
-  return 1024 + stages * stage_bytes + (size_t)4 * rows_alloc * (16 + 4) + rows_alloc * 4;
+size_t head_smem_bytes(int rows_alloc) {
+  return 1024 + (size_t)head_ep_bytes(rows_alloc) + head_ring_bytes(rows_alloc);
 }
 
 }  // namespace
@@ -642,8 +642,9 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     uint8_t* hc = W.hidden_c;
     int32_t* rm = W.row_map;
     int32_t* nr = W.n_rows;
-    void* args[] = {(void*)&hid, (void*)&masked, (void*)&bk, (void*)&rb, (void*)&hc,
-                    (void*)&rm,  (void*)&nr,     (void*)&entropy, (void*)&token};
+    void* args[] = {(void*)&hid, (void*)&masked,  (void*)&bk,    (void*)&rb,
+                    (void*)&hc,  (void*)&rm,      (void*)&nr,    (void*)&entropy,
+                    (void*)&token};
     s = launch_pdl((const void*)compact_rows_kernel, dim3(p.rows_alloc), dim3(256), 0, st, args,
                    "compact_rows_kernel launch");
     if (s != SBD_OK) return s;
@@ -679,14 +680,13 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.H = p.H;
     a.rows_alloc = p.rows_alloc;
     a.n_tiles = (p.V + kBM - 1) / kBM;
-    a.boxes = head_boxes(p.H, p.rows_alloc);
-    a.stages = head_stages(p.rows_alloc, a.boxes);
+    a.ring_bytes = head_ring_bytes(p.rows_alloc);
     a.n_acc = 2 * p.rows_alloc <= 512 ? 2 : 1;
     uint32_t cols = 32;
     while (cols < (uint32_t)(a.n_acc * p.rows_alloc)) cols <<= 1;
     a.tmem_cols = cols;
     a.tau = tau;
-    const size_t smem = head_smem_bytes(p.rows_alloc, a.stages, a.boxes);
+    const size_t smem = head_smem_bytes(p.rows_alloc);
     e = cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");

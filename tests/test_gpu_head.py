@@ -63,7 +63,8 @@ def test_tiny_f32_config(sbd):
 
 @pytest.mark.parametrize("B,k,V,H", [(1, 1, 1000, 256), (1, 16, 4096 + 5, 512), (2, 16, 3000, 128),
                                      (3, 7, 777, 64), (16, 16, 2100, 256), (1, 17, 500, 128),
-                                     (10, 30, 999, 64), (16, 32, 1500, 128)])
+                                     (10, 30, 999, 64), (16, 32, 1500, 128),
+                                     (2, 16, 40000, 1024), (1, 8, 60013, 512)])
 @pytest.mark.parametrize("tau", [0.0, 1.0])
 def test_bf16_shapes(sbd, B, k, V, H, tau):
     w = gen.shrink(gen.get_workload("llama8b_k16"), batch=B, block_k=k, vocab=V, hidden=H,

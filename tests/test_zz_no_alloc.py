@@ -26,8 +26,8 @@ def sbd():
 
 
 def test_oversized_shape_is_rejected_before_any_launch(sbd):
-    # fp32, 256 rows of 8192 hidden: 8 MiB of compacted rows > 4 MiB scratch
-    d = sbd.HeadDesc(16, 16, 8192, 512, sbd.SBD_DTYPE_F32)
+    # fp32, 256 rows of 16384 hidden: 16 MiB of compacted rows > 8 MiB scratch
+    d = sbd.HeadDesc(16, 16, 16384, 512, sbd.SBD_DTYPE_F32)
     a = 1 << 20                                   # never dereferenced
     st = sbd.lib.sbd_head_entropy_sample_noalloc(ctypes.byref(d), a, a, a, a, 1.0, a, a, None)
     assert st == sbd.SBD_ERR_UNSUPPORTED
