@@ -12,10 +12,12 @@
 //                        W and hidden tiles into a shared-memory ring with
 //                        TMA; one thread issues tcgen05.mma into a
 //                        double-buffered fp32 accumulator in tensor memory;
-//                        four epilogue warps read it back with tcgen05.ld and
-//                        reduce every logit column to running statistics
-//                        (max, sum of exponentials, entropy numerator, best
-//                        Gumbel score and id) -- logits never reach HBM;
+//                        eight epilogue warps (two per TMEM lane quadrant,
+//                        alternate 16-column chunks) read it back with
+//                        tcgen05.ld and reduce every logit column to running
+//                        statistics (max, sum of exponentials, entropy
+//                        numerator, best Gumbel score and id) -- logits never
+//                        reach HBM;
 //   head_f32_kernel      (fp32) the same reduction over exact fp32 FMAs;
 //   head_combine_kernel  merges the per-CTA statistics of each row into the
 //                        entropy (nats) and the token.
@@ -48,7 +50,22 @@ constexpr int kMaxStages = 16;
 #ifndef SBD_HEAD_EVICT_FIRST
 #define SBD_HEAD_EVICT_FIRST 1
 #endif
-constexpr int kHeadThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+// Epilogue warps: 4 or 8 (warps 2, 3, ...; warp w reads TMEM lanes of
+// quadrant w % 4, and the warps of one quadrant take alternate 16-column
+// chunks).
+#ifndef SBD_HEAD_EPI_WARPS
+#define SBD_HEAD_EPI_WARPS 8
+#endif
+constexpr int kEpiWarps = SBD_HEAD_EPI_WARPS;
+// Chunks of Gumbel noise an epilogue warp keeps in flight ahead of the one
+// it reduces (loads from HBM take longer than the reduction of one chunk).
+#ifndef SBD_HEAD_G_AHEAD
+#define SBD_HEAD_G_AHEAD 2
+#endif
+constexpr int kGAhead = SBD_HEAD_G_AHEAD;
+static_assert(kEpiWarps == 4 || kEpiWarps == 8, "4 or 8 epilogue warps");
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kHeadThreads = 64 + kEpiThreads;   // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -152,25 +169,80 @@ __device__ __forceinline__ RowStats warp_column_stats(float z, bool valid, float
   return st;
 }
 
-// Reduces 16 columns over the 32 lanes of a warp at once (lane = vocabulary
-// row): at each level a lane keeps half of its columns and merges in the
-// partner lane's copy of them, so 16 + 8 + 4 + 2 + 1 merges replace
-// 16 x 5 full warp reductions.  On return st[0] of lanes 2c and 2c + 1
-// holds column c.
-__device__ __forceinline__ void butterfly16(RowStats (&st)[16], int lane) {
+// Statistics of 16 logit columns over the 32 vocabulary rows of a warp
+// (lane = row, vocabulary id v0 + lane; z the logits, g the Gumbel noise).
+// Two passes: the column maxima of z log2(e) and of the Gumbel score
+// z + tau g go through a transposed max butterfly (16 + 8 + 4 + 2 + 1 steps
+// instead of 16 x 5); every lane then takes exp2 of its logits against the
+// column maxima, and the sums of the exponentials and of their entropy terms
+// go through the same butterfly with additions.  The best id is the lowest
+// lane that reaches the column's best score (ties to the lowest id).  On
+// return lanes 2c and 2c + 1 hold column c.
+__device__ __forceinline__ RowStats chunk16_stats(const float (&z)[16], const float (&g)[16],
+                                                  bool valid, float tau, int v0, int lane) {
+  float s[16], sc[16], ms[16], mb[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    s[j] = valid ? z[j] * kLog2e : -INFINITY;
+    sc[j] = valid ? fmaf(tau, g[j], z[j]) : -INFINITY;
+    ms[j] = s[j];
+    mb[j] = sc[j];
+  }
 #pragma unroll
   for (int lvl = 0; lvl < 4; ++lvl) {
-    const int b = 16 >> lvl;           // lane bit of this level
-    const int half = 8 >> lvl;         // columns kept
+    const int b = 16 >> lvl;
+    const int half = 8 >> lvl;
     const bool upper = (lane & b) != 0;
 #pragma unroll
     for (int i = 0; i < half; ++i) {
-      const RowStats keep = upper ? st[i + half] : st[i];
-      const RowStats send = upper ? st[i] : st[i + half];
-      st[i] = rowstats_merge(keep, shfl_xor_stats(send, b));
+      const float ks = upper ? ms[i + half] : ms[i];
+      const float ss = upper ? ms[i] : ms[i + half];
+      const float kb = upper ? mb[i + half] : mb[i];
+      const float sb = upper ? mb[i] : mb[i + half];
+      ms[i] = fmaxf(ks, __shfl_xor_sync(0xffffffffu, ss, b));
+      mb[i] = fmaxf(kb, __shfl_xor_sync(0xffffffffu, sb, b));
     }
   }
-  st[0] = rowstats_merge(st[0], shfl_xor_stats(st[0], 1));
+  ms[0] = fmaxf(ms[0], __shfl_xor_sync(0xffffffffu, ms[0], 1));
+  mb[0] = fmaxf(mb[0], __shfl_xor_sync(0xffffffffu, mb[0], 1));
+
+  const int my_col = (lane >> 1) & 15;
+  unsigned my_hits = 0u;
+  float e[16], t[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float m = __shfl_sync(0xffffffffu, ms[0], 2 * j);
+    const float best = __shfl_sync(0xffffffffu, mb[0], 2 * j);
+    const float d = s[j] - m;                  // <= 0 on valid lanes
+    e[j] = valid ? exp2f(d) : 0.f;
+    t[j] = valid ? e[j] * d : 0.f;
+    const unsigned hits = __ballot_sync(0xffffffffu, valid && sc[j] == best);
+    if (my_col == j) my_hits = hits;
+  }
+#pragma unroll
+  for (int lvl = 0; lvl < 4; ++lvl) {
+    const int b = 16 >> lvl;
+    const int half = 8 >> lvl;
+    const bool upper = (lane & b) != 0;
+#pragma unroll
+    for (int i = 0; i < half; ++i) {
+      const float ke = upper ? e[i + half] : e[i];
+      const float se = upper ? e[i] : e[i + half];
+      const float kt = upper ? t[i + half] : t[i];
+      const float st = upper ? t[i] : t[i + half];
+      e[i] = ke + __shfl_xor_sync(0xffffffffu, se, b);
+      t[i] = kt + __shfl_xor_sync(0xffffffffu, st, b);
+    }
+  }
+  e[0] += __shfl_xor_sync(0xffffffffu, e[0], 1);
+  t[0] += __shfl_xor_sync(0xffffffffu, t[0], 1);
+  RowStats r;
+  r.m = ms[0];
+  r.S = e[0];
+  r.T = t[0];
+  r.best = mb[0];
+  r.idx = my_hits ? v0 + __ffs(my_hits) - 1 : 0x7fffffff;
+  return r;
 }
 
 struct StatsRef {
@@ -294,6 +366,10 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int stage_bytes = boxes * (kABytes + b_box);     // [A boxes | B boxes]
   int stages = a.ring_bytes / stage_bytes;
   if (stages > kMaxStages) stages = kMaxStages;
+  // Epilogue warps with a chunk of 16 columns to reduce, per TMEM quadrant;
+  // the others skip the tile loop.
+  const int n_chunks = (R + 15) / 16;
+  const int n_sub = n_chunks < kEpiWarps / 4 ? (n_chunks > 0 ? n_chunks : 1) : kEpiWarps / 4;
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
       mbar_init(&full_bar[s], 1);
@@ -301,13 +377,13 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tmem_full[i], 1);
-      mbar_init(&tmem_empty[i], 4);     // one arrival per epilogue warp
+      mbar_init(&tmem_empty[i], 4 * n_sub);   // one arrival per working epilogue warp
     }
     fence_mbar_init();
   }
   if (warp >= 2) {
     const int te = threadIdx.x - 64;
-    for (int i = te; i < a.rows_alloc; i += 128) {
+    for (int i = te; i < a.rows_alloc; i += kEpiThreads) {
       rmap[i] = i < R ? a.row_map[i] : 0;
       for (int w = 0; w < 4; ++w) store_stats(wstats[w], i, rowstats_empty());
     }
@@ -397,31 +473,45 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       }
     } else {
       // ------------------------------------------------ epilogue warps
-      const int ew = warp - 2;                 // 0..3
       const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
+      const int sub = (warp - 2) / 4;          // chunks sub, sub + n_sub, ... of 16 columns
       const bool noisy = a.tau != 0.f && a.gumbel != nullptr;
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
-      for (int tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x, ++local) {
+      for (int tile = blockIdx.x; sub < n_sub && tile < a.n_tiles; tile += gridDim.x, ++local) {
         const int acc = a.n_acc == 2 ? (local & 1) : 0;
         const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
-        const int v = tile * kBM + quad * 32 + lane;
+        const int v0 = tile * kBM + quad * 32;
+        const int v = v0 + lane;
         const bool valid = v < a.V;
         const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)(acc * a.rows_alloc);
-        // Gumbel noise of the first 16 columns is loaded while the MMAs run,
-        // that of the next 16 while the current ones are reduced.
-        float g[16], g_next[16];
+        // Gumbel noise of the first kGAhead chunks is loaded while the MMAs
+        // run; each chunk's reduction then loads the chunk kGAhead further on.
+        const int stride = 16 * n_sub;
+        const int c_first = 16 * sub;
+        float gq[kGAhead][16];
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          g_next[j] = (noisy && valid && j < R) ? __ldg(a.gumbel + (size_t)rmap[j] * a.V + v) : 0.f;
-        if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
-        tc_fence_after();
-        for (int c0 = 0; c0 < R; c0 += 16) {
+        for (int d = 0; d < kGAhead; ++d)
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            g[j] = g_next[j];
-            const int cn = c0 + 16 + j;
-            g_next[j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            const int cn = c_first + d * stride + j;
+            gq[d][j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+          }
+        if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
+        tc_fence_after();
+        for (int c0 = c_first; c0 < R; c0 += stride) {
+          float g[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) g[j] = gq[0][j];
+#pragma unroll
+          for (int d = 0; d + 1 < kGAhead; ++d)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) gq[d][j] = gq[d + 1][j];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int cn = c0 + kGAhead * stride + j;
+            gq[kGAhead - 1][j] =
+                (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
           }
           uint32_t r[16];
           tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
@@ -429,21 +519,18 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
           float z[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
-          RowStats st[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j) st[j] = lane_stats(z[j], valid, g[j], a.tau, v);
-          butterfly16(st, lane);
+          const RowStats st = chunk16_stats(z, g, valid, a.tau, v0, lane);
           const int col = c0 + ((lane >> 1) & 15);
           if ((lane & 1) == 0 && col < R)
-            store_stats(wstats[ew], col, rowstats_merge(load_stats(wstats[ew], col), st[0]));
+            store_stats(wstats[quad], col, rowstats_merge(load_stats(wstats[quad], col), st));
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tmem_empty[acc]);
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
       const int te = threadIdx.x - 64;
-      for (int col = te; col < R; col += 128) {
+      for (int col = te; col < R; col += kEpiThreads) {
         RowStats s = load_stats(wstats[0], col);
         for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats[w], col));
         const size_t o = (size_t)blockIdx.x * a.rows_alloc + col;
