@@ -17,7 +17,13 @@ Readings of points the paper leaves open (each listed in the design notes):
   * sampling is Gumbel-max on z + tau * g (tau = 0: greedy, the paper's
     temperature-0 setting), ties to the lowest vocabulary id;
   * EB rule with the inequality exactly as printed (<=), gamma = 0 allowed,
-    equal entropies ordered by block position.
+    equal entropies ordered by block position;
+  * confidence c^i = max_v p_v of softmax(z) at temperature 1; confidence
+    orders are descending, equal confidences ordered by block position;
+  * Factor rule: c^n is the n-th largest confidence, n the largest count in
+    1..|M| with (n + 1) c^n < f, and n = 1 when no count qualifies (a step
+    unmasks at least one token); the complement reading (n + 1)(1 - c^n) < f
+    is provided beside it.
 
 Pins (what each function is checked against, none of it itself) live in
 tests/test_oracle_*.py; no function here is "parity unpinned".
@@ -132,6 +138,15 @@ def entropy(z_row: np.ndarray) -> float:
     return float(terms.sum())
 
 
+def confidence(z_row: np.ndarray) -> float:
+    """Confidence c^i = max_v p(x_i = v | x_<t, x_J) of a position's
+    predicted marginal, p = softmax(z) (Appendix "Sampling algorithm": the
+    Factor rule and the confidence error proxy of the general EB-Sampler).
+    With the max subtracted: max_v p_v = 1 / sum_v exp(z_v - max z)."""
+    z = np.asarray(z_row, dtype=np.float64)
+    return float(1.0 / np.exp(z - z.max()).sum())
+
+
 def sample_token(z_row: np.ndarray, g_row, tau: float) -> int:
     """Gumbel-max sample: argmax_v (z_v + tau * g_v); tau = 0 (or no noise)
     is greedy decoding, the paper's temperature-0 setting (Sec. 3.1).  For
@@ -145,7 +160,7 @@ def sample_token(z_row: np.ndarray, g_row, tau: float) -> int:
 
 
 def head_entropy_sample(hidden, w_store, w_dtype, masked, gumbel, tau,
-                        rows=None, vocab_chunk: int = 8192):
+                        rows=None, vocab_chunk: int = 8192, with_confidence=False):
     """Per block position: entropy (nats) and sampled token of the masked
     positions' predicted marginals p_theta(x_{t+i} | x_<t; x_hat) (Eqs. 6-7,
     Algorithm 3 "compute probabilities").  Position t+i predicts its own
@@ -156,25 +171,28 @@ def head_entropy_sample(hidden, w_store, w_dtype, masked, gumbel, tau,
     token -1.  `rows`, if given, restricts the work to those (b, i) pairs
     (the others are left as +inf / -1).  Returns (entropy [B,k] f64,
     token [B,k] int32, z dict {(b,i): z_row}) -- z is returned for test
-    diagnostics (top-2 gaps)."""
+    diagnostics (top-2 gaps).  with_confidence=True appends confidence
+    [B,k] f64 (0 at unmasked positions)."""
     B, k, H = hidden.shape
     ent = np.full((B, k), np.inf, dtype=np.float64)
     tok = np.full((B, k), MASK_TOKEN, dtype=np.int32)
+    conf = np.zeros((B, k), dtype=np.float64)
     if rows is None:
         rows = [(b, i) for b in range(B) for i in range(k) if masked[b, i]]
     else:
         rows = [(b, i) for (b, i) in rows if masked[b, i]]
     if not rows:
-        return ent, tok, {}
+        return (ent, tok, {}, conf) if with_confidence else (ent, tok, {})
     hr = np.stack([hidden[b, i] for (b, i) in rows])
     z = logits(hr, w_store, w_dtype, vocab_chunk)
     zs = {}
     for n, (b, i) in enumerate(rows):
         ent[b, i] = entropy(z[n])
+        conf[b, i] = confidence(z[n])
         g = None if gumbel is None else gumbel[b, i]
         tok[b, i] = sample_token(z[n], g, tau)
         zs[(b, i)] = z[n]
-    return ent, tok, zs
+    return (ent, tok, zs, conf) if with_confidence else (ent, tok, zs)
 
 
 # ------------------------------------------------------------- EB select
@@ -237,3 +255,95 @@ def eb_prefix_margins(entropy_row_sorted, gamma: float):
         prefix += float(entropy_row_sorted[j - 1])
         out.append(abs(prefix - gamma))
     return out
+
+
+# ------------------------------------------------- other selection rules
+
+def eb_general_accept_count(entropies_in_order, gamma: float) -> int:
+    """General EB-Sampler bound (Appendix "Sampling algorithm", the general
+    form of Eq. 3): with the masked positions taken in the order i_1, i_2,
+    ... of the error proxy, s >= 1 is the largest count with
+        sum_{j<=s} H_{i_j} - max_{j'<=s} H_{i_j'} <= gamma,
+    capped at |M|.  Sums in float64.  For non-negative entropies the left
+    side never decreases as s grows (a new term adds H and raises the max by
+    at most H), so the largest such s is found by walking the order until
+    the first count that breaks the bound."""
+    n = len(entropies_in_order)
+    if n == 0:
+        return 0
+    s = 1
+    total = float(entropies_in_order[0])
+    top = total
+    for j in range(1, n):                  # candidate s = j + 1
+        h = float(entropies_in_order[j])
+        total += h
+        top = max(top, h)
+        if total - top <= gamma:
+            s = j + 1
+        else:
+            break
+    return s
+
+
+def factor_accept_count(confidences_desc, f: float, complement: bool = False) -> int:
+    """Factor parallel decoding (Appendix "Sampling algorithm"): with the
+    masked confidences sorted descending c^1 >= c^2 >= ..., unmask the first
+    n, n the largest count in 1..|M| with
+        (n + 1) c^n < f                 (c^n read as the n-th confidence),
+    or, with complement=True, (n + 1) (1 - c^n) < f.  When no count
+    qualifies n = 1, so that every step unmasks a token; 0 when |M| = 0.
+    The literal condition need not hold for a prefix of counts, so every
+    count is tested."""
+    n_m = len(confidences_desc)
+    if n_m == 0:
+        return 0
+    best = 1
+    for n in range(1, n_m + 1):
+        c = float(confidences_desc[n - 1])
+        lhs = (n + 1) * ((1.0 - c) if complement else c)
+        if lhs < f:
+            best = n
+    return best
+
+
+SELECT_RULES = ("eb_entropy", "eb_confidence", "factor", "factor_complement")
+
+
+def select_step(entropy_bk, confidence_bk, token_bk, masked_bk, block_tokens_bk,
+                rule: str, threshold: float):
+    """One unmasking step under one of the selection rules of the paper
+    (Algorithm 3 "unmask tokens", with the rule of Eq. 3 or of the Appendix
+    "Sampling algorithm"):
+      eb_entropy         Eq. 3 (same as eb_select; threshold = gamma);
+      eb_confidence      positions ordered by confidence, descending, and the
+                         general EB bound (threshold = gamma);
+      factor             confidence order, (n + 1) c^n < f (threshold = f);
+      factor_complement  confidence order, (n + 1)(1 - c^n) < f.
+    Ties of the ordering key go to the lower block position.  Returns the
+    same tuple as eb_select."""
+    if rule not in SELECT_RULES:
+        raise ValueError(rule)
+    if rule == "eb_entropy":
+        return eb_select(entropy_bk, token_bk, masked_bk, block_tokens_bk, threshold)
+    B, k = masked_bk.shape
+    new_masked = np.array(masked_bk, dtype=np.uint8, copy=True)
+    new_bt = np.array(block_tokens_bk, dtype=np.int32, copy=True)
+    n_un = np.zeros(B, dtype=np.int32)
+    accepted = []
+    orders = []
+    for b in range(B):
+        M = [i for i in range(k) if masked_bk[b, i]]
+        order = sorted(M, key=lambda i: (-float(confidence_bk[b, i]), i))
+        if rule == "eb_confidence":
+            s = eb_general_accept_count([entropy_bk[b, i] for i in order], threshold)
+        else:
+            s = factor_accept_count([confidence_bk[b, i] for i in order], threshold,
+                                    complement=(rule == "factor_complement"))
+        acc = set(order[:s])
+        for i in acc:
+            new_bt[b, i] = token_bk[b, i]
+            new_masked[b, i] = 0
+        n_un[b] = s
+        accepted.append(acc)
+        orders.append(order)
+    return new_masked, new_bt, n_un, accepted, orders

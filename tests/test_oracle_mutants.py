@@ -174,3 +174,114 @@ def test_eb_descending_sort_is_caught(monkeypatch):
     monkeypatch.setattr(oracle, "eb_select", desc)
     pins = [(TE.test_worked_example, ()), (TE.test_ties_ordered_by_position, ())]
     assert any(_fails(fn, *args) for fn, args in pins)
+
+
+# ------------------------------------------------- confidence and other rules
+from tests import test_oracle_select as TS   # noqa: E402
+
+
+def _patch(monkeypatch, name, fn):
+    monkeypatch.setattr(so, name, fn)
+    monkeypatch.setattr(oracle, name, fn)
+
+
+def _conf_mean_shift(z_row):
+    z = np.asarray(z_row, dtype=np.float64)
+    return float(1.0 / np.exp(z - z.mean()).sum())   # the mean subtracted, not the max
+
+
+def _conf_without_shift(z_row):
+    z = np.asarray(z_row, dtype=np.float64)
+    return float(1.0 / np.exp(z).sum())            # max subtracted nowhere
+
+
+@pytest.mark.parametrize("mutant", [_conf_mean_shift, _conf_without_shift])
+def test_confidence_mutants_are_caught(monkeypatch, mutant):
+    _patch(monkeypatch, "confidence", mutant)
+    pins = [(TS.test_uniform_logits_confidence_is_one_over_v, (7,)),
+            (TS.test_two_point_confidence_is_logistic, (1.0, -1.0)),
+            (TS.test_confidence_matches_softmax_and_bounds_entropy, ())]
+    assert any(_fails(fn, *args) for fn, args in pins)
+
+
+def _general_without_max(H_in_order, gamma):
+    n = len(H_in_order)
+    if n == 0:
+        return 0
+    s, total = 1, float(H_in_order[0])
+    for j in range(1, n):
+        total += float(H_in_order[j])
+        if total <= gamma:                         # the max term dropped
+            s = j + 1
+        else:
+            break
+    return s
+
+
+def _general_exclusive_prefix(H_in_order, gamma):
+    n = len(H_in_order)
+    if n == 0:
+        return 0
+    s, prefix = 1, 0.0
+    for j in range(1, n):
+        prefix += float(H_in_order[j - 1])         # Eq. 3's sum, in a non-sorted order
+        if prefix <= gamma:
+            s = j + 1
+        else:
+            break
+    return s
+
+
+@pytest.mark.parametrize("mutant", [_general_without_max, _general_exclusive_prefix])
+def test_general_bound_mutants_are_caught(monkeypatch, mutant):
+    _patch(monkeypatch, "eb_general_accept_count", mutant)
+    pins = [(TS.test_confidence_proxy_worked_example, ()), (TS.test_running_max_matters, ()),
+            (TS.test_general_bound_invariants, ())]
+    assert any(_fails(fn, *args) for fn, args in pins)
+
+
+def _factor_off_by_one(confidences_desc, f, complement=False):
+    n_m = len(confidences_desc)
+    if n_m == 0:
+        return 0
+    best = 1
+    for n in range(1, n_m + 1):
+        c = float(confidences_desc[n - 1])
+        if n * ((1.0 - c) if complement else c) < f:   # n instead of n + 1
+            best = n
+    return best
+
+
+def _factor_first_failure(confidences_desc, f, complement=False):
+    n_m = len(confidences_desc)
+    if n_m == 0:
+        return 0
+    best = 1
+    for n in range(1, n_m + 1):
+        c = float(confidences_desc[n - 1])
+        if (n + 1) * ((1.0 - c) if complement else c) < f:
+            best = n
+        else:
+            break                                   # stops at the first failing count
+    return best
+
+
+@pytest.mark.parametrize("mutant", [_factor_off_by_one, _factor_first_failure])
+def test_factor_mutants_are_caught(monkeypatch, mutant):
+    _patch(monkeypatch, "factor_accept_count", mutant)
+    pins = [(TS.test_factor_worked_examples, ()),
+            (TS.test_factor_constant_confidence_closed_form, (0.3, 1.0))]
+    assert any(_fails(fn, *args) for fn, args in pins)
+
+
+def test_ascending_confidence_order_is_caught(monkeypatch):
+    real = so.select_step
+
+    def asc(entropy_bk, confidence_bk, token_bk, masked_bk, block_tokens_bk, rule, thr):
+        return real(entropy_bk, -np.asarray(confidence_bk), token_bk, masked_bk,
+                    block_tokens_bk, rule, thr)
+
+    monkeypatch.setattr(oracle, "select_step", asc)
+    pins = [(TS.test_confidence_proxy_worked_example, ()),
+            (TS.test_factor_select_takes_a_confidence_prefix, ())]
+    assert any(_fails(fn, *args) for fn, args in pins)
