@@ -126,6 +126,24 @@ sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden
                                    size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * sbd_head_entropy_sample plus the confidence of every masked position, for
+ * the confidence-ordered selection rules of the Appendix "Sampling
+ * algorithm" (Factor decoding; EB-Sampler with the confidence proxy):
+ *   confidence = max_v p_v,  p = softmax(z) at temperature 1,
+ * computed from the same merged statistics as the entropy (1 / sum_v
+ * exp(z_v - max z)).  Unmasked positions get confidence = 0.
+ *   confidence [B, k] fp32 out; every other argument, the workspace (size
+ *   from sbd_head_entropy_sample_workspace_size) and the errors are those of
+ *   sbd_head_entropy_sample.
+ * ---------------------------------------------------------------------- */
+sbd_status sbd_head_entropy_confidence_sample(const sbd_head_desc* desc, const void* hidden,
+                                              const void* w, const uint8_t* masked,
+                                              const float* gumbel, float tau, float* entropy,
+                                              float* confidence, int32_t* token,
+                                              void* workspace, size_t workspace_bytes,
+                                              void* stream);
+
+/* ------------------------------------------------------------------------
  * No-allocation variant of sbd_head_entropy_sample.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory -- a host framework that owns the whole device memory pool,
@@ -172,6 +190,45 @@ sbd_status sbd_head_entropy_sample_noalloc(const sbd_head_desc* desc, const void
 sbd_status sbd_eb_select(int32_t batch, int32_t block_k, const float* entropy,
                          const int32_t* token, float gamma, uint8_t* masked,
                          int32_t* block_tokens, int32_t* n_unmasked, void* stream);
+
+/* ------------------------------------------------------------------------
+ * One unmasking step under a selectable rule (Algorithm 3 "unmask"; the
+ * rules of Eq. 3 and of the Appendix "Sampling algorithm").  Per sequence b
+ * the masked positions are ordered by the rule's key (ties to the lower
+ * position), the first s accepted, their tokens committed and their flags
+ * cleared, exactly as in sbd_eb_select:
+ *   SBD_SELECT_EB_ENTROPY          entropy ascending; s of Eq. 3 with
+ *                                  threshold = gamma.  Identical to
+ *                                  sbd_eb_select (confidence not read).
+ *   SBD_SELECT_EB_CONFIDENCE       confidence descending; s >= 1 the largest
+ *                                  count with  sum_{j<=s} H_{i_j} -
+ *                                  max_{j'<=s} H_{i_j'} <= gamma  (the
+ *                                  general EB bound), capped at |M|.
+ *   SBD_SELECT_FACTOR              confidence descending, c^1 >= c^2 >= ...;
+ *                                  s the largest n in 1..|M| with
+ *                                  (n + 1) c^n < f  (threshold = f), s = 1
+ *                                  when no n qualifies.
+ *   SBD_SELECT_FACTOR_COMPLEMENT   as FACTOR with (n + 1)(1 - c^n) < f.
+ * Sums, maxima and products in fp32.  A NaN key sorts last.
+ *
+ *   entropy [B, k] fp32, confidence [B, k] fp32 (may be NULL for
+ *   SBD_SELECT_EB_ENTROPY), token [B, k] int32   inputs
+ *   masked [B, k] uint8, block_tokens [B, k] int32 (-1 = mask)   in/out
+ *   n_unmasked [B] int32 out (may be NULL)
+ * Supported: 1 <= k <= 32; threshold finite and >= 0.  An unknown rule is
+ * SBD_ERR_INVALID_ARG.
+ * ---------------------------------------------------------------------- */
+typedef enum {
+  SBD_SELECT_EB_ENTROPY = 0,
+  SBD_SELECT_EB_CONFIDENCE = 1,
+  SBD_SELECT_FACTOR = 2,
+  SBD_SELECT_FACTOR_COMPLEMENT = 3
+} sbd_select_rule;
+
+sbd_status sbd_select(int32_t rule, int32_t batch, int32_t block_k, const float* entropy,
+                      const float* confidence, const int32_t* token, float threshold,
+                      uint8_t* masked, int32_t* block_tokens, int32_t* n_unmasked,
+                      void* stream);
 
 /* Status name ("SBD_OK", ...). Never NULL. */
 const char* sbd_status_string(sbd_status status);

@@ -33,6 +33,10 @@ SBD_DEVERR_CACHE_LEN = 1
 SBD_DEVERR_TIMEOUT = 2
 SBD_DEVERR_ROWS = 4
 SBD_HEAD_NOALLOC_MAX_SCRATCH = 8 << 20
+SBD_SELECT_EB_ENTROPY = 0
+SBD_SELECT_EB_CONFIDENCE = 1
+SBD_SELECT_FACTOR = 2
+SBD_SELECT_FACTOR_COMPLEMENT = 3
 
 # Every symbol include/sbd.h declares.
 EXPORTS = (
@@ -41,7 +45,9 @@ EXPORTS = (
     "sbd_head_entropy_sample_workspace_size",
     "sbd_head_entropy_sample",
     "sbd_head_entropy_sample_noalloc",
+    "sbd_head_entropy_confidence_sample",
     "sbd_eb_select",
+    "sbd_select",
     "sbd_status_string",
     "sbd_last_error",
     "sbd_device_error",
@@ -87,8 +93,13 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_head_entropy_sample_noalloc.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp,
                                                     f32, vp, vp, vp]
     lib.sbd_head_entropy_sample_noalloc.restype = ctypes.c_int
+    lib.sbd_head_entropy_confidence_sample.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp,
+                                                       f32, vp, vp, vp, vp, sz, vp]
+    lib.sbd_head_entropy_confidence_sample.restype = ctypes.c_int
     lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
     lib.sbd_eb_select.restype = ctypes.c_int
+    lib.sbd_select.argtypes = [i32, i32, i32, vp, vp, vp, f32, vp, vp, vp, vp]
+    lib.sbd_select.restype = ctypes.c_int
     lib.sbd_status_string.argtypes = [ctypes.c_int]
     lib.sbd_status_string.restype = ctypes.c_char_p
     lib.sbd_last_error.argtypes = []
@@ -218,6 +229,34 @@ def sbd_head_entropy_sample(hidden, w, masked, gumbel, tau: float, entropy=None,
     return entropy, token
 
 
+def sbd_head_entropy_confidence_sample(hidden, w, masked, gumbel, tau: float, entropy=None,
+                                       confidence=None, token=None, *, workspace=None,
+                                       stream=None):
+    """sbd_head_entropy_sample plus confidence = max_v p_v of every masked
+    position (0 at unmasked ones), for the confidence-ordered selection
+    rules.  Returns (entropy [B,k] fp32, confidence [B,k] fp32, token [B,k]
+    int32)."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, gumbel=gumbel, entropy=entropy,
+               confidence=confidence, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    B, k, _ = hidden.shape
+    if entropy is None:
+        entropy = torch.empty((B, k), dtype=torch.float32, device=hidden.device)
+    if confidence is None:
+        confidence = torch.empty((B, k), dtype=torch.float32, device=hidden.device)
+    if token is None:
+        token = torch.empty((B, k), dtype=torch.int32, device=hidden.device)
+    d = head_desc(hidden, w)
+    ws = _workspace(lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(d)), hidden.device,
+                    workspace)
+    _check(lib.sbd_head_entropy_confidence_sample(
+        ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked), _ptr(gumbel), float(tau),
+        _ptr(entropy), _ptr(confidence), _ptr(token), _ptr(ws), _nbytes(ws), _stream(stream)))
+    return entropy, confidence, token
+
+
 def sbd_head_entropy_sample_noalloc(hidden, w, masked, gumbel, tau: float, entropy, token, *,
                                     stream=None):
     """sbd_head_entropy_sample for callers that cannot allocate device
@@ -248,6 +287,24 @@ def sbd_eb_select(entropy, token, gamma: float, masked, block_tokens, n_unmasked
         n_unmasked = torch.empty(B, dtype=torch.int32, device=masked.device)
     _check(lib.sbd_eb_select(B, k, _ptr(entropy), _ptr(token), float(gamma), _ptr(masked),
                              _ptr(block_tokens), _ptr(n_unmasked), _stream(stream)))
+    return n_unmasked
+
+
+def sbd_select(rule: int, entropy, confidence, token, threshold: float, masked, block_tokens,
+               n_unmasked=None, *, stream=None):
+    """One unmasking step under `rule` (SBD_SELECT_*: Eq. 3, the general EB
+    bound in confidence order, or the Factor rule); threshold is gamma or f.
+    Updates masked and block_tokens in place; returns n_unmasked [B] int32.
+    confidence may be None for SBD_SELECT_EB_ENTROPY."""
+    torch = _torch()
+    _need_cuda(entropy=entropy, confidence=confidence, token=token, masked=masked,
+               block_tokens=block_tokens, n_unmasked=n_unmasked)
+    B, k = masked.shape
+    if n_unmasked is None:
+        n_unmasked = torch.empty(B, dtype=torch.int32, device=masked.device)
+    _check(lib.sbd_select(int(rule), B, k, _ptr(entropy), _ptr(confidence), _ptr(token),
+                          float(threshold), _ptr(masked), _ptr(block_tokens), _ptr(n_unmasked),
+                          _stream(stream)))
     return n_unmasked
 
 

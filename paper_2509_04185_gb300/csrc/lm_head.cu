@@ -20,7 +20,8 @@
 //                        reach HBM;
 //   head_f32_kernel      (fp32) the same reduction over exact fp32 FMAs;
 //   head_combine_kernel  merges the per-CTA statistics of each row into the
-//                        entropy (nats) and the token.
+//                        entropy (nats), the token and, when asked for, the
+//                        confidence max_v p_v = 1 / S.
 #include <math.h>
 
 #include "sbd_internal.cuh"
@@ -269,7 +270,8 @@ __global__ void __launch_bounds__(256)
 compact_rows_kernel(const uint8_t* __restrict__ hidden, const uint8_t* __restrict__ masked,
                     int BK, int row_bytes, uint8_t* __restrict__ hidden_c,
                     int32_t* __restrict__ row_map, int32_t* __restrict__ n_rows,
-                    float* __restrict__ entropy, int32_t* __restrict__ token) {
+                    float* __restrict__ entropy, int32_t* __restrict__ token,
+                    float* __restrict__ confidence) {
   grid_dependency_wait();
   grid_dependents_launch();
   const int row = blockIdx.x;
@@ -294,6 +296,7 @@ compact_rows_kernel(const uint8_t* __restrict__ hidden, const uint8_t* __restric
       if (t == 0) {
         entropy[row] = INFINITY;
         token[row] = -1;
+        if (confidence) confidence[row] = 0.f;
       }
     }
   } else {
@@ -611,7 +614,7 @@ __global__ void __launch_bounds__(128)
 head_combine_kernel(const float4* __restrict__ part_msTb, const int32_t* __restrict__ part_idx,
                     int n_parts, int rows_alloc, const int32_t* __restrict__ row_map,
                     const int32_t* __restrict__ n_rows, float* __restrict__ entropy,
-                    int32_t* __restrict__ token) {
+                    int32_t* __restrict__ token, float* __restrict__ confidence) {
   grid_dependency_wait();
   const int r = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -641,6 +644,8 @@ head_combine_kernel(const float4* __restrict__ part_msTb, const int32_t* __restr
     const int row = row_map[r];
     entropy[row] = kLn2 * (log2f(s.S) - s.T / s.S);
     token[row] = s.idx;
+    // the largest probability is the max term's: 2^0 / S
+    if (confidence) confidence[row] = 1.f / s.S;
   }
 }
 
@@ -717,7 +722,7 @@ size_t head_workspace_bytes(const HeadPlan& p) { return head_ws_layout(p, nullpt
 
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
-                       int32_t* token, void* ws, cudaStream_t st) {
+                       float* confidence, int32_t* token, void* ws, cudaStream_t st) {
   const int BK = p.B * p.k;
   if (BK == 0) return SBD_OK;
   HeadWs W = head_ws_layout(p, ws);
@@ -731,7 +736,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     int32_t* nr = W.n_rows;
     void* args[] = {(void*)&hid, (void*)&masked,  (void*)&bk,    (void*)&rb,
                     (void*)&hc,  (void*)&rm,      (void*)&nr,    (void*)&entropy,
-                    (void*)&token};
+                    (void*)&token, (void*)&confidence};
     s = launch_pdl((const void*)compact_rows_kernel, dim3(p.rows_alloc), dim3(256), 0, st, args,
                    "compact_rows_kernel launch");
     if (s != SBD_OK) return s;
@@ -802,8 +807,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     int np = p.n_ctas, ra = p.rows_alloc;
     const int32_t* rm = W.row_map;
     const int32_t* nr = W.n_rows;
-    void* args[] = {(void*)&pm, (void*)&pi, (void*)&np, (void*)&ra,
-                    (void*)&rm, (void*)&nr, (void*)&entropy, (void*)&token};
+    void* args[] = {(void*)&pm, (void*)&pi, (void*)&np,      (void*)&ra,   (void*)&rm,
+                    (void*)&nr, (void*)&entropy, (void*)&token, (void*)&confidence};
     s = launch_pdl((const void*)head_combine_kernel, dim3((p.rows_alloc + 3) / 4), dim3(128), 0,
                    st, args, "head_combine_kernel launch");
     if (s != SBD_OK) return s;

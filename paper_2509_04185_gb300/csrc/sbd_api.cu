@@ -215,10 +215,14 @@ size_t sbd_head_entropy_sample_workspace_size(const sbd_head_desc* desc) {
   return sbd::head_workspace_bytes(sbd::head_plan(*desc));
 }
 
-sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden, const void* w,
-                                   const uint8_t* masked, const float* gumbel, float tau,
-                                   float* entropy, int32_t* token, void* workspace,
-                                   size_t workspace_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+
+sbd_status head_call(const sbd_head_desc* desc, const void* hidden, const void* w,
+                     const uint8_t* masked, const float* gumbel, float tau, float* entropy,
+                     float* confidence, int32_t* token, void* workspace, size_t workspace_bytes,
+                     void* stream) {
   sbd_status s = check_head_desc(desc);
   if (s != SBD_OK) return s;
   if (!(isfinite(tau) && tau >= 0.f))
@@ -230,6 +234,8 @@ sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden
     if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
     if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
   }
+  if (confidence && !aligned16(confidence))
+    return fail(SBD_ERR_INVALID_ARG, "confidence is not 16-byte aligned");
   if (tau != 0.f && !gumbel)
     return fail(SBD_ERR_INVALID_ARG, "gumbel is NULL but tau != 0");
   if (gumbel && !aligned16(gumbel))
@@ -241,24 +247,68 @@ sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden
                 workspace ? workspace_bytes : (size_t)0);
   if (!aligned16(workspace)) return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
   return sbd::head_launch(p, hidden, w, masked, tau == 0.f ? nullptr : gumbel, tau, entropy,
-                          token, workspace, (cudaStream_t)stream);
+                          confidence, token, workspace, (cudaStream_t)stream);
 }
 
-sbd_status sbd_eb_select(int32_t batch, int32_t block_k, const float* entropy,
-                         const int32_t* token, float gamma, uint8_t* masked,
-                         int32_t* block_tokens, int32_t* n_unmasked, void* stream) {
+sbd_status select_call(int32_t rule, int32_t batch, int32_t block_k, const float* entropy,
+                       const float* confidence, const int32_t* token, float threshold,
+                       uint8_t* masked, int32_t* block_tokens, int32_t* n_unmasked,
+                       void* stream) {
+  if (rule < SBD_SELECT_EB_ENTROPY || rule > SBD_SELECT_FACTOR_COMPLEMENT)
+    return fail(SBD_ERR_INVALID_ARG, "unknown selection rule %d", rule);
   if (batch < 0 || block_k < 1)
     return fail(SBD_ERR_INVALID_ARG, "bad sizes: batch=%d block_k=%d", batch, block_k);
   if (block_k > 32) return fail(SBD_ERR_UNSUPPORTED, "block_k %d > 32", block_k);
-  if (!(isfinite(gamma) && gamma >= 0.f))
-    return fail(SBD_ERR_INVALID_ARG, "gamma must be finite and >= 0");
+  if (!(isfinite(threshold) && threshold >= 0.f))
+    return fail(SBD_ERR_INVALID_ARG, "%s must be finite and >= 0",
+                rule <= SBD_SELECT_EB_CONFIDENCE ? "gamma" : "f");
   if (batch == 0) return SBD_OK;
   const void* ptrs[] = {entropy, token, masked, block_tokens};
   const char* names[] = {"entropy", "token", "masked", "block_tokens"};
   for (int i = 0; i < 4; ++i)
     if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
-  return sbd::eb_launch(batch, block_k, entropy, token, gamma, masked, block_tokens, n_unmasked,
-                        (cudaStream_t)stream);
+  if (rule != SBD_SELECT_EB_ENTROPY && !confidence)
+    return fail(SBD_ERR_INVALID_ARG, "confidence is NULL but rule %d orders by confidence", rule);
+  return sbd::select_launch(rule, batch, block_k, entropy, confidence, token, threshold, masked,
+                            block_tokens, n_unmasked, (cudaStream_t)stream);
+}
+
+}  // namespace
+
+extern "C" {
+
+sbd_status sbd_head_entropy_sample(const sbd_head_desc* desc, const void* hidden, const void* w,
+                                   const uint8_t* masked, const float* gumbel, float tau,
+                                   float* entropy, int32_t* token, void* workspace,
+                                   size_t workspace_bytes, void* stream) {
+  return head_call(desc, hidden, w, masked, gumbel, tau, entropy, nullptr, token, workspace,
+                   workspace_bytes, stream);
+}
+
+sbd_status sbd_head_entropy_confidence_sample(const sbd_head_desc* desc, const void* hidden,
+                                              const void* w, const uint8_t* masked,
+                                              const float* gumbel, float tau, float* entropy,
+                                              float* confidence, int32_t* token,
+                                              void* workspace, size_t workspace_bytes,
+                                              void* stream) {
+  if (!confidence) return fail(SBD_ERR_INVALID_ARG, "confidence is NULL");
+  return head_call(desc, hidden, w, masked, gumbel, tau, entropy, confidence, token, workspace,
+                   workspace_bytes, stream);
+}
+
+sbd_status sbd_eb_select(int32_t batch, int32_t block_k, const float* entropy,
+                         const int32_t* token, float gamma, uint8_t* masked,
+                         int32_t* block_tokens, int32_t* n_unmasked, void* stream) {
+  return select_call(SBD_SELECT_EB_ENTROPY, batch, block_k, entropy, nullptr, token, gamma,
+                     masked, block_tokens, n_unmasked, stream);
+}
+
+sbd_status sbd_select(int32_t rule, int32_t batch, int32_t block_k, const float* entropy,
+                      const float* confidence, const int32_t* token, float threshold,
+                      uint8_t* masked, int32_t* block_tokens, int32_t* n_unmasked,
+                      void* stream) {
+  return select_call(rule, batch, block_k, entropy, confidence, token, threshold, masked,
+                     block_tokens, n_unmasked, stream);
 }
 
 const char* sbd_status_string(sbd_status status) {

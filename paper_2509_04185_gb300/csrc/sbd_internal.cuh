@@ -50,11 +50,12 @@ HeadPlan head_plan(const sbd_head_desc& d);
 size_t head_workspace_bytes(const HeadPlan& p);
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
-                       int32_t* token, void* ws, cudaStream_t st);
+                       float* confidence, int32_t* token, void* ws, cudaStream_t st);
 
-sbd_status eb_launch(int B, int k, const float* entropy, const int32_t* token, float gamma,
-                     uint8_t* masked, int32_t* block_tokens, int32_t* n_unmasked,
-                     cudaStream_t st);
+// rule: an sbd_select_rule value (SBD_SELECT_EB_ENTROPY for sbd_eb_select)
+sbd_status select_launch(int rule, int B, int k, const float* entropy, const float* confidence,
+                         const int32_t* token, float threshold, uint8_t* masked,
+                         int32_t* block_tokens, int32_t* n_unmasked, cudaStream_t st);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 

@@ -116,6 +116,39 @@ def test_eb_rejects_bad_arguments(sbd):
     assert sbd.lib.sbd_eb_select(0, 4, None, None, 0.1, None, None, None, None) == sbd.SBD_OK
 
 
+def test_select_rejects_bad_arguments(sbd):
+    a = 1 << 20
+    for rule in (-1, 4, 99):
+        assert sbd.lib.sbd_select(rule, 1, 4, a, a, a, 0.1, a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
+        assert b"rule" in sbd.lib.sbd_last_error()
+    for rule in (sbd.SBD_SELECT_EB_CONFIDENCE, sbd.SBD_SELECT_FACTOR,
+                 sbd.SBD_SELECT_FACTOR_COMPLEMENT):
+        # confidence-ordered rules need the confidence
+        assert sbd.lib.sbd_select(rule, 1, 4, a, None, a, 0.1, a, a, a, None) == \
+            sbd.SBD_ERR_INVALID_ARG
+        assert sbd.lib.sbd_select(rule, 1, 33, a, a, a, 0.1, a, a, a, None) == \
+            sbd.SBD_ERR_UNSUPPORTED
+        for thr in (-0.5, float("nan"), float("inf")):
+            assert sbd.lib.sbd_select(rule, 1, 4, a, a, a, thr, a, a, a, None) == \
+                sbd.SBD_ERR_INVALID_ARG
+    assert sbd.lib.sbd_select(sbd.SBD_SELECT_FACTOR, 0, 4, None, None, None, 1.0, None, None,
+                              None, None) == sbd.SBD_OK
+
+
+def test_confidence_head_rejects_bad_arguments(sbd):
+    a = 1 << 20
+    d = sbd.HeadDesc(1, 16, 4096, 128256, sbd.SBD_DTYPE_BF16)
+    f = sbd.lib.sbd_head_entropy_confidence_sample
+    assert f(ctypes.byref(d), a, a, a, a, 1.0, a, None, a, a, 1 << 30, None) == \
+        sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(d), a, a, a, a, 1.0, a, a + 4, a, a, 1 << 30, None) == \
+        sbd.SBD_ERR_INVALID_ARG
+    assert b"confidence" in sbd.lib.sbd_last_error()
+    d = sbd.HeadDesc(32, 17, 4096, 128256, sbd.SBD_DTYPE_BF16)      # 544 rows > 512
+    assert f(ctypes.byref(d), a, a, a, a, 1.0, a, a, a, a, 1 << 30, None) == \
+        sbd.SBD_ERR_UNSUPPORTED
+
+
 def test_binding_refuses_cpu_tensors(sbd):
     import torch
     x = torch.zeros(1, 4, 4, 64)
