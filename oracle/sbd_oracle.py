@@ -20,6 +20,10 @@ Readings of points the paper leaves open (each listed in the design notes):
     equal entropies ordered by block position;
   * confidence c^i = max_v p_v of softmax(z) at temperature 1; confidence
     orders are descending, equal confidences ordered by block position;
+  * the first iteration of a block after the previous one carries the
+    previous block's tokens as n_causal causal rows ahead of the new block
+    (their keys and values then enter the cache); the new block's rows see
+    them like the rest of the cache;
   * Factor rule: c^n is the n-th largest confidence, n the largest count in
     1..|M| with (n + 1) c^n < f, and n = 1 when no count qualifies (a step
     unmasks at least one token); the complement reading (n + 1)(1 - c^n) < f
@@ -58,12 +62,20 @@ def inference_mask_allows(q_idx: int, kv_idx: int, causal_point: int) -> bool:
     return (kv_idx <= q_idx) or (causal_point <= q_idx)
 
 
-def block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None):
+def block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None,
+                    n_causal: int = 0):
     """Block attention of one SBD forward (Eq. 5; Fig. 3 mask).
 
     Block query row i of sequence b attends to the L_b cached keys (the exact
     KV cache of x_<t, causal among themselves and all in the past of the
     block) and to all k block keys (bidirectional inside the block).
+
+    n_causal > 0 is the first iteration of a block after the previous one
+    (Algorithm 3, "first iteration and t >= k"): the forward then carries
+    the n_causal tokens of the previous block, whose keys and values still
+    have to enter the cache, ahead of the new block.  Under the inference
+    mask with its causal point at the new block, block row i < n_causal sees
+    the cache and block keys j <= i; rows i >= n_causal see every key.
 
     q [B,k,Hq,D]; k_cache, v_cache [B,Lmax,Hkv,D]; cache_len [B];
     k_blk, v_blk [B,k,Hkv,D]; all float64.  Returns o [B,k,Hq,D] float64.
@@ -81,11 +93,33 @@ def block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None):
             keys = np.concatenate([k_cache[b, :L, hk, :], k_blk[b, :, hk, :]], axis=0)
             vals = np.concatenate([v_cache[b, :L, hk, :], v_blk[b, :, hk, :]], axis=0)
             s = (q[b, :, hq, :] @ keys.T) * scale            # [k, L+k]
+            for i in range(min(n_causal, k)):                 # causal rows of the block
+                s[i, L + i + 1:] = -np.inf
             s = s - s.max(axis=1, keepdims=True)
             p = np.exp(s)
             p = p / p.sum(axis=1, keepdims=True)
             out[b, :, hq, :] = p @ vals
     return out
+
+
+def kv_append(k_cache, v_cache, cache_len, k_rows, v_rows):
+    """The keys and values of the n tokens the cache lacks (the previous
+    block, processed causally in the first iteration of the next one,
+    Algorithm 3) are written at positions L_b .. L_b + n - 1 of the cache.
+    k_rows, v_rows [B,n,Hkv,D].  Returns new (k_cache, v_cache, cache_len);
+    the inputs are not modified."""
+    kc = np.array(k_cache, copy=True)
+    vc = np.array(v_cache, copy=True)
+    n = k_rows.shape[1]
+    lens = np.array(cache_len, dtype=np.int64, copy=True)
+    for b in range(kc.shape[0]):
+        L = int(lens[b])
+        if L + n > kc.shape[1]:
+            raise ValueError("cache overflow")
+        kc[b, L:L + n] = k_rows[b]
+        vc[b, L:L + n] = v_rows[b]
+        lens[b] = L + n
+    return kc, vc, lens
 
 
 def masked_sequence_attention(q_seq, k_seq, v_seq, causal_point, scale=None):

@@ -25,7 +25,7 @@ def _rand_inputs(B, k, Hq, Hkv, D, L, seed, lens=None):
     return q, kc, vc, np.asarray(lens, dtype=np.int32), kb, vb
 
 
-def _explicit_mask_attention(q, kc, vc, lens, kb, vb, scale=None):
+def _explicit_mask_attention(q, kc, vc, lens, kb, vb, scale=None, n_causal=0):
     """Full-sequence attention, one head at a time, where every position of
     the sequence x_<t ; x_hat_t..x_hat_{t+k-1} is a query and the mask is an
     explicit [T, T] boolean matrix built from the paper's inference predicate
@@ -43,7 +43,7 @@ def _explicit_mask_attention(q, kc, vc, lens, kb, vb, scale=None):
         mask = np.zeros((T, T), dtype=bool)
         for qi in range(T):
             for kv in range(T):
-                mask[qi, kv] = oracle.inference_mask_allows(qi, kv, L)
+                mask[qi, kv] = oracle.inference_mask_allows(qi, kv, L + n_causal)
         for hq in range(Hq):
             hk = hq // G
             K = np.concatenate([kc[b, :L, hk], kb[b, :, hk]])
@@ -172,3 +172,71 @@ def test_scale_override():
     np.testing.assert_allclose(a, b, atol=1e-12)
     ref = _explicit_mask_attention(q, kc, vc, lens, kb, vb, scale=0.5)
     np.testing.assert_allclose(a, ref, atol=1e-12)
+
+
+# ------------------------------------------- first iteration: causal prefix rows
+
+@pytest.mark.parametrize("k,n_causal,L", [(4, 2, 5), (6, 3, 0), (2, 1, 3), (8, 4, 6), (3, 3, 4)])
+def test_causal_prefix_rows_equal_explicit_mask(k, n_causal, L):
+    q, kc, vc, lens, kb, vb = _rand_inputs(2, k, 4, 2, 8, max(L, 1), seed=100 + k * 7 + n_causal,
+                                           lens=[L, max(L - 2, 0)])
+    got = oracle.block_attention(q, kc, vc, lens, kb, vb, n_causal=n_causal)
+    ref = _explicit_mask_attention(q, kc, vc, lens, kb, vb, n_causal=n_causal)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+
+
+def test_all_causal_block_is_torch_causal_prefill():
+    # every block row causal: plain causal attention over cache + block
+    B, k, Hq, Hkv, D, L = 2, 5, 4, 2, 16, 6
+    q, kc, vc, lens, kb, vb = _rand_inputs(B, k, Hq, Hkv, D, L, seed=77)
+    got = oracle.block_attention(q, kc, vc, lens, kb, vb, n_causal=k)
+    G = Hq // Hkv
+    for b in range(B):
+        K = torch.from_numpy(np.concatenate([kc[b], kb[b]]))          # [L+k, Hkv, D]
+        V = torch.from_numpy(np.concatenate([vc[b], vb[b]]))
+        Q = torch.from_numpy(q[b])                                      # [k, Hq, D]
+        allowed = torch.ones(k, L + k, dtype=torch.bool)
+        allowed[:, L:] = torch.tril(torch.ones(k, k, dtype=torch.bool))
+        for hq in range(Hq):
+            ref = torch.nn.functional.scaled_dot_product_attention(
+                Q[:, hq][None], K[:, hq // G][None], V[:, hq // G][None], attn_mask=allowed)[0]
+            np.testing.assert_allclose(got[b, :, hq], ref.numpy(), rtol=0, atol=1e-12)
+
+
+def test_bidirectional_rows_equal_block_after_append():
+    # The new block's rows of a first-iteration forward (2k rows, the first k
+    # causal) see what a plain block forward sees once the previous block is
+    # in the cache.
+    B, k, Hq, Hkv, D, L = 2, 4, 4, 2, 8, 9
+    rng = np.random.default_rng(5)
+    q2 = rng.standard_normal((B, 2 * k, Hq, D))
+    kc = rng.standard_normal((B, L + k, Hkv, D))
+    vc = rng.standard_normal((B, L + k, Hkv, D))
+    kb2 = rng.standard_normal((B, 2 * k, Hkv, D))
+    vb2 = rng.standard_normal((B, 2 * k, Hkv, D))
+    lens = np.array([L, L - 3], dtype=np.int32)
+    two_k = oracle.block_attention(q2, kc, vc, lens, kb2, vb2, n_causal=k)
+    kc2, vc2, lens2 = oracle.kv_append(kc, vc, lens, kb2[:, :k], vb2[:, :k])
+    assert list(lens2) == [L + k, L - 3 + k]
+    one = oracle.block_attention(q2[:, k:], kc2, vc2, lens2, kb2[:, k:], vb2[:, k:])
+    np.testing.assert_allclose(two_k[:, k:], one, rtol=0, atol=1e-12)
+
+
+def test_kv_append_writes_only_the_new_rows():
+    rng = np.random.default_rng(2)
+    kc = rng.standard_normal((2, 10, 2, 4))
+    vc = rng.standard_normal((2, 10, 2, 4))
+    kr = rng.standard_normal((2, 3, 2, 4))
+    vr = rng.standard_normal((2, 3, 2, 4))
+    lens = np.array([4, 7])
+    kc0, lens0 = kc.copy(), lens.copy()
+    k2, v2, l2 = oracle.kv_append(kc, vc, lens, kr, vr)
+    assert list(l2) == [7, 10]
+    np.testing.assert_array_equal(k2[0, 4:7], kr[0])
+    np.testing.assert_array_equal(v2[1, 7:10], vr[1])
+    np.testing.assert_array_equal(k2[0, :4], kc[0, :4])
+    np.testing.assert_array_equal(k2[0, 7:], kc[0, 7:])
+    np.testing.assert_array_equal(kc, kc0)         # inputs unmodified
+    np.testing.assert_array_equal(lens, lens0)
+    with pytest.raises(ValueError):
+        oracle.kv_append(kc, vc, np.array([8, 0]), kr, vr)

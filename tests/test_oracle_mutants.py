@@ -285,3 +285,39 @@ def test_ascending_confidence_order_is_caught(monkeypatch):
     pins = [(TS.test_confidence_proxy_worked_example, ()),
             (TS.test_factor_select_takes_a_confidence_prefix, ())]
     assert any(_fails(fn, *args) for fn, args in pins)
+
+
+# ------------------------------------------------ causal prefix rows (first iteration)
+
+def _prefix_mutant(shift):
+    """block_attention whose causal rows see block keys j <= i + shift."""
+    def f(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None, n_causal=0):
+        B, k, Hq, D = q.shape
+        G = Hq // k_cache.shape[2]
+        sc = 1.0 / np.sqrt(D) if scale is None else scale
+        out = np.zeros_like(q)
+        for b in range(B):
+            L = int(cache_len[b])
+            for hq in range(Hq):
+                hk = hq // G
+                keys = np.concatenate([k_cache[b, :L, hk], k_blk[b, :, hk]])
+                vals = np.concatenate([v_cache[b, :L, hk], v_blk[b, :, hk]])
+                s = q[b, :, hq] @ keys.T * sc
+                for i in range(min(n_causal, k)):
+                    s[i, max(L + i + 1 + shift, L + 1):] = -np.inf
+                p = np.exp(s - s.max(axis=1, keepdims=True))
+                out[b, :, hq] = (p / p.sum(axis=1, keepdims=True)) @ vals
+        return out
+    return f
+
+
+def _prefix_ignored(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale=None, n_causal=0):
+    return so.block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, scale)
+
+
+@pytest.mark.parametrize("mutant", [_prefix_mutant(-1), _prefix_mutant(1), _prefix_ignored])
+def test_causal_prefix_mutants_are_caught(monkeypatch, mutant):
+    monkeypatch.setattr(oracle, "block_attention", mutant)
+    pins = [(TA.test_causal_prefix_rows_equal_explicit_mask, (4, 2, 5)),
+            (TA.test_all_causal_block_is_torch_causal_prefill, ())]
+    assert all(_fails(fn, *args) for fn, args in pins)
