@@ -92,6 +92,29 @@ sbd_status sbd_block_attention(const sbd_attn_desc* desc, const void* q,
                                size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Block attention of the first iteration of a block after the previous one
+ * (Algorithm 3, "first iteration and t >= k"; the inference mask of the
+ * FlexAttention appendix listing with its causal point at the new block).
+ * The forward carries the n_causal tokens of the previous block, which the
+ * cache does not hold yet, as the leading block rows:
+ *   block row i <  n_causal  sees the cached keys and block keys j <= i;
+ *   block row i >= n_causal  sees the cached keys and all block keys;
+ * and the keys/values of rows i < n_causal are written into the caches at
+ * positions cache_len[b] + i.  cache_len itself is not changed: the caller
+ * advances it by n_causal once the call has completed.  Arguments, layouts,
+ * workspace and errors are those of sbd_block_attention, except that
+ * k_cache / v_cache are written (only at the n_causal new positions), and
+ * 0 <= n_causal <= block_k (else SBD_ERR_INVALID_ARG).  A sequence with
+ * cache_len[b] + n_causal > max_cache_len gets no append and sets
+ * SBD_DEVERR_CACHE_LEN.  n_causal = 0 is sbd_block_attention.
+ * ---------------------------------------------------------------------- */
+sbd_status sbd_block_attention_causal_prefix(const sbd_attn_desc* desc, int32_t n_causal,
+                                             const void* q, void* k_cache, void* v_cache,
+                                             const int32_t* cache_len, const void* k_blk,
+                                             const void* v_blk, void* out, void* workspace,
+                                             size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * LM head + entropy + Gumbel-max sample (Eqs. 6-7; Algorithm 3 "compute
  * probabilities"), over the MASKED block positions only.  For masked
  * position (b, i) with hidden row h = hidden[b, i, :]:

@@ -42,6 +42,7 @@ SBD_SELECT_FACTOR_COMPLEMENT = 3
 EXPORTS = (
     "sbd_block_attention_workspace_size",
     "sbd_block_attention",
+    "sbd_block_attention_causal_prefix",
     "sbd_head_entropy_sample_workspace_size",
     "sbd_head_entropy_sample",
     "sbd_head_entropy_sample_noalloc",
@@ -85,6 +86,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_block_attention.argtypes = [ctypes.POINTER(AttnDesc), vp, vp, vp, vp, vp, vp, vp,
                                         vp, sz, vp]
     lib.sbd_block_attention.restype = ctypes.c_int
+    lib.sbd_block_attention_causal_prefix.argtypes = [ctypes.POINTER(AttnDesc), i32, vp, vp, vp,
+                                                      vp, vp, vp, vp, vp, sz, vp]
+    lib.sbd_block_attention_causal_prefix.restype = ctypes.c_int
     lib.sbd_head_entropy_sample_workspace_size.argtypes = [ctypes.POINTER(HeadDesc)]
     lib.sbd_head_entropy_sample_workspace_size.restype = sz
     lib.sbd_head_entropy_sample.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp, f32, vp,
@@ -203,6 +207,29 @@ def sbd_block_attention(q, k_cache, v_cache, cache_len, k_blk, v_blk, out=None, 
     _check(lib.sbd_block_attention(ctypes.byref(d), _ptr(q), _ptr(k_cache), _ptr(v_cache),
                                    _ptr(cache_len), _ptr(k_blk), _ptr(v_blk), _ptr(out),
                                    _ptr(ws), _nbytes(ws), _stream(stream)))
+    return out
+
+
+def sbd_block_attention_causal_prefix(q, k_cache, v_cache, cache_len, k_blk, v_blk,
+                                      n_causal: int, out=None, *, scale: float = 0.0,
+                                      num_splits: int = 0, workspace=None, stream=None):
+    """First iteration of a block after the previous one (Algorithm 3): block
+    rows i < n_causal (the previous block's tokens) are causal among the
+    block keys and their keys/values are written into k_cache / v_cache at
+    cache_len[b] + i (cache_len is not changed); the other rows see every
+    key.  Shapes as sbd_block_attention; returns out."""
+    torch = _torch()
+    _need_cuda(q=q, k_cache=k_cache, v_cache=v_cache, cache_len=cache_len, k_blk=k_blk,
+               v_blk=v_blk, out=out)
+    if cache_len.dtype != torch.int32:
+        raise TypeError("cache_len must be int32")
+    if out is None:
+        out = torch.empty_like(q)
+    d = attn_desc(q, k_cache, scale, num_splits)
+    ws = _workspace(lib.sbd_block_attention_workspace_size(ctypes.byref(d)), q.device, workspace)
+    _check(lib.sbd_block_attention_causal_prefix(
+        ctypes.byref(d), int(n_causal), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len),
+        _ptr(k_blk), _ptr(v_blk), _ptr(out), _ptr(ws), _nbytes(ws), _stream(stream)))
     return out
 
 

@@ -12,12 +12,19 @@
 //     split and are copied in by the same warp;
 //   * compute warps own 16 query rows each and, when M is small, a slice of
 //     every key tile; S = Q K^T and O += P V run on bf16 mma.sync with fp32
-//     accumulators in registers; the mask (cache key < L_b, block key < k)
-//     is applied to the score registers; the online softmax keeps its row
+//     accumulators in registers; the mask (cache key < L_b, block key < k,
+//     block key j <= i for a causal block row i < n_causal) is applied to
+//     the score registers; the online softmax keeps its row
 //     max and sum per thread and reduces them across the 4 threads of a row
 //     with shuffles;
 //   * with more than one split, each CTA writes its normalised partial
 //     output and log-sum-exp, merged by attn_combine_kernel.
+//
+// First iteration of a block after the previous one (Algorithm 3, "first
+// iteration and t >= k"): the leading n_causal block rows are the previous
+// block's tokens, causal among themselves, and their keys/values are written
+// into the cache at L_b .. L_b + n_causal - 1 by the warp that copies the
+// block tile in (one CTA per (KV head, sequence)).
 //
 // The fp32 variant (attn_f32_kernel) is a plain SIMT kernel with fp32 FMAs
 // throughout, used for fp32 inputs.
@@ -88,7 +95,9 @@ struct AttnArgs {
   float* part_o;             // [B, Hkv, S, M, D] (splits > 1)
   float* part_lse;           // [B, Hkv, S, M]
   int* err;
-  int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG, stages;
+  __nv_bfloat16* kc_app;     // writable caches for the causal rows' keys/values, or NULL
+  __nv_bfloat16* vc_app;
+  int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG, stages, n_causal;
   float scale_log2;
 };
 
@@ -171,6 +180,13 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
             const size_t off = (((size_t)b * a.k + j) * a.Hkv + hkv) * D + cc * 8;
             kv = *reinterpret_cast<const uint4*>(a.kb + off);
             vv = *reinterpret_cast<const uint4*>(a.vb + off);
+            if (a.kc_app && j < a.n_causal && len + a.n_causal <= a.Lmax) {
+              // a causal row enters the cache (positions >= len are read by
+              // no split of this call, or masked and zeroed where they are)
+              const size_t dst = (((size_t)b * a.Lmax + len + j) * a.Hkv + hkv) * D + cc * 8;
+              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv;
+              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv;
+            }
           }
           const int h = cc / 8, c8 = cc % 8;
           const uint32_t ka = swz(kbase + h * kSubBytes, j, c8);
@@ -182,6 +198,8 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
                        "r"(vv.z), "r"(vv.w)
                        : "memory");
         }
+        if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
+          record_error(a.err, SBD_DEVERR_CACHE_LEN);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&full_bar[stage]);
@@ -237,6 +255,12 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
       }
       const bool block_tile = t >= n_cache_tiles;
       const int valid = block_tile ? a.k : min(kTileKeys, len - t * kTileKeys);
+      // causal rows of the block see the block keys j <= i only
+      int valid0 = valid, valid1 = valid;
+      if (block_tile) {
+        if (r0 / a.G < a.n_causal) valid0 = r0 / a.G + 1;
+        if (r1 / a.G < a.n_causal) valid1 = r1 / a.G + 1;
+      }
       const uint32_t kbase = smem_base + stage * kStageBytes;
       const uint32_t vbase = kbase + kSub * kSubBytes;
       const int key0 = kg * NK;
@@ -265,9 +289,8 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
           const int key = key0 + n * 8 + qc + e;
-          const bool vis = key < valid;
-          s[n][e] = vis ? s[n][e] * a.scale_log2 : -INFINITY;
-          s[n][2 + e] = vis ? s[n][2 + e] * a.scale_log2 : -INFINITY;
+          s[n][e] = key < valid0 ? s[n][e] * a.scale_log2 : -INFINITY;
+          s[n][2 + e] = key < valid1 ? s[n][2 + e] * a.scale_log2 : -INFINITY;
           mx0 = fmaxf(mx0, s[n][e]);
           mx1 = fmaxf(mx1, s[n][2 + e]);
         }
@@ -484,7 +507,8 @@ attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
                 const float* __restrict__ vc, const int32_t* __restrict__ lens,
                 const float* __restrict__ kb, const float* __restrict__ vb,
                 float* __restrict__ out, int* err, int k, int Hq, int Hkv, int D, int Lmax,
-                float scale_log2) {
+                float scale_log2, int n_causal, float* __restrict__ kc_app,
+                float* __restrict__ vc_app) {
   __shared__ float qs[128];
   __shared__ float ps[128];
   __shared__ float red[4];
@@ -499,8 +523,21 @@ attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
   }
   const float* qrow = q + (((size_t)b * k + i) * Hq + hq) * D;
   if (tid < D) qs[tid] = qrow[tid];
+  // The first CTA of each KV head writes a causal row's key and value into
+  // the cache; the attention below reads cache positions < len only.
+  if (kc_app && i < n_causal && hq % G == 0 && tid < D) {
+    if (len + n_causal <= Lmax) {
+      const size_t dst = (((size_t)b * Lmax + len + i) * Hkv + hkv) * D + tid;
+      const size_t src = (((size_t)b * k + i) * Hkv + hkv) * D + tid;
+      kc_app[dst] = kb[src];
+      vc_app[dst] = vb[src];
+    } else if (tid == 0 && i == 0) {
+      sbd_dev::record_error(err, SBD_DEVERR_CACHE_LEN);
+    }
+  }
   __syncthreads();
-  const int total = len + k;
+  // causal rows of the block see the block keys j <= i only
+  const int total = len + (i < n_causal ? i + 1 : k);
   float m = -INFINITY, l = 0.f, acc = 0.f;   // acc: output element d = tid
   for (int c0 = 0; c0 < total; c0 += 128) {
     const int u = c0 + tid;
@@ -577,6 +614,7 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
   p.Lmax = d.max_cache_len;
   p.M = p.G * p.k;
   p.bf16 = d.dtype == SBD_DTYPE_BF16;
+  p.n_causal = 0;
   const float scale = d.scale != 0.f ? d.scale : 1.0f / sqrtf((float)d.head_dim);
   p.scale_log2 = scale * kLog2e;
   const int tiles = (p.Lmax + kTileKeys - 1) / kTileKeys + 1;
@@ -613,7 +651,7 @@ static size_t attn_smem_bytes(const AttnPlan& p) {
 
 sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const void* vc,
                        const int32_t* lens, const void* kb, const void* vb, void* out, void* ws,
-                       cudaStream_t st) {
+                       void* kc_app, void* vc_app, cudaStream_t st) {
   if (p.B == 0) return SBD_OK;
   int* err = device_error_word();
   if (!p.bf16) {
@@ -622,9 +660,13 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
     float* of = (float*)out;
     int k = p.k, Hq = p.Hq, Hkv = p.Hkv, D = p.D, Lmax = p.Lmax;
     float sl2 = p.scale_log2;
-    void* args[] = {(void*)&qf, (void*)&kcf, (void*)&vcf, (void*)&lens, (void*)&kbf,
-                    (void*)&vbf, (void*)&of,  (void*)&err, (void*)&k,    (void*)&Hq,
-                    (void*)&Hkv, (void*)&D,   (void*)&Lmax, (void*)&sl2};
+    int nc = p.n_causal;
+    float* kca = (float*)kc_app;
+    float* vca = (float*)vc_app;
+    void* args[] = {(void*)&qf,  (void*)&kcf, (void*)&vcf,  (void*)&lens, (void*)&kbf,
+                    (void*)&vbf, (void*)&of,  (void*)&err,  (void*)&k,    (void*)&Hq,
+                    (void*)&Hkv, (void*)&D,   (void*)&Lmax, (void*)&sl2,  (void*)&nc,
+                    (void*)&kca, (void*)&vca};
     return launch_pdl((const void*)attn_f32_kernel, dim3(p.k, p.Hq, p.B), dim3(128), 0, st, args,
                       "attn_f32_kernel launch");
   }
@@ -660,6 +702,9 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.MT = p.MT;
   a.KG = p.KG;
   a.stages = p.stages;
+  a.n_causal = p.n_causal;
+  a.kc_app = (__nv_bfloat16*)kc_app;
+  a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
   a.part_o = (float*)ws;
@@ -668,7 +713,8 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   // Up to 16 packed rows the mma.sync kernel measures faster (the tcgen05
   // kernel pads every tile to 128 rows); above, tcgen05.
   if (SBD_ATTN_TC && p.M > 16) {
-    s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, st);
+    s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, kc_app, vc_app,
+                       st);
     if (s != SBD_OK) return s;
   } else {
   const int NW = a.MT * a.KG;

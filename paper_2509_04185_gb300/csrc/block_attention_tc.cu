@@ -16,7 +16,7 @@
 // the tensor memory and one thread issues the MMAs, computing S_{j+1} while
 // the softmax of tile j runs; warps 2-5 are the softmax: thread = row, it
 // reads its 64 scores with tcgen05.ld, applies the mask (cache key < L_b,
-// block key < k) and the scale, and writes P_j = 2^(s - m_ref) as bf16 into
+// block key < k, or j <= i for a causal block row i < n_causal) and the scale, and writes P_j = 2^(s - m_ref) as bf16 into
 // shared memory.  The reference max m_ref only moves (and O is rescaled in
 // tensor memory) when the running max exceeds it by more than 2^8, which
 // keeps every P entry <= 256; l and O use the same reference, so the result
@@ -141,7 +141,9 @@ struct TcArgs {
   float* part_o;
   float* part_lse;
   int* err;
-  int B, k, Hq, Hkv, G, M, Lmax, splits;
+  __nv_bfloat16* kc_app;     // writable caches for the causal rows' keys/values, or NULL
+  __nv_bfloat16* vc_app;
+  int B, k, Hq, Hkv, G, M, Lmax, splits, n_causal;
   float scale_log2;
 };
 
@@ -267,10 +269,19 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
             const size_t off = (((size_t)b * a.k + row) * a.Hkv + hkv) * D + cc * 8;
             kv = *reinterpret_cast<const uint4*>(a.kb + off);
             vv = *reinterpret_cast<const uint4*>(a.vb + off);
+            if (a.kc_app && row < a.n_causal && len + a.n_causal <= a.Lmax) {
+              // a causal row enters the cache (positions >= len are read by
+              // no split of this call, or masked and zeroed where they are)
+              const size_t dst = (((size_t)b * a.Lmax + len + row) * a.Hkv + hkv) * D + cc * 8;
+              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv;
+              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv;
+            }
           }
           st_shared_v4(swz(ks + (cc / 8) * kKVSub, row, cc % 8), kv);
           st_shared_v4(swz(vs + (cc / 8) * kKVSub, row, cc % 8), vv);
         }
+        if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
+          record_error(a.err, SBD_DEVERR_CACHE_LEN);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&kv_full[stage]);
@@ -356,7 +367,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     bool ok = true;
     for (int j = 0; j < n && ok; ++j) {
       const int t = t_begin + j;
-      const int valid = t < n_cache_tiles ? min(kTileKeys, len - t * kTileKeys) : a.k;
+      int valid = t < n_cache_tiles ? min(kTileKeys, len - t * kTileKeys) : a.k;
+      // causal rows of the block see the block keys j <= i only
+      if (t >= n_cache_tiles && row / a.G < a.n_causal) valid = row / a.G + 1;
       if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) {
         ok = false;
         break;
@@ -529,7 +542,8 @@ size_t attn_tc_smem_bytes(int D) {
 
 sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
                           const void* q, const int32_t* lens, const void* kb, const void* vb,
-                          void* out, float* part_o, float* part_lse, cudaStream_t st) {
+                          void* out, float* part_o, float* part_lse, void* kc_app,
+                          void* vc_app, cudaStream_t st) {
   TcArgs a;
   a.q = (const __nv_bfloat16*)q;
   a.kb = (const __nv_bfloat16*)kb;
@@ -547,6 +561,9 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.M = p.M;
   a.Lmax = p.Lmax;
   a.splits = p.splits;
+  a.n_causal = p.n_causal;
+  a.kc_app = (__nv_bfloat16*)kc_app;
+  a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t smem = attn_tc_smem_bytes(p.D);
   const void* fn = p.D == 128 ? (const void*)attn_tc_kernel<128> : (const void*)attn_tc_kernel<64>;

@@ -176,6 +176,32 @@ sbd_status check_head_desc(const sbd_head_desc* d) {
   return SBD_OK;
 }
 
+sbd_status attn_call(const sbd_attn_desc* desc, int n_causal, const void* q, const void* k_cache,
+                     const void* v_cache, const int32_t* cache_len, const void* k_blk,
+                     const void* v_blk, void* out, void* workspace, size_t workspace_bytes,
+                     void* kc_app, void* vc_app, void* stream) {
+  sbd_status s = check_attn_desc(desc);
+  if (s != SBD_OK) return s;
+  if (desc->batch == 0) return SBD_OK;
+  const void* ptrs[] = {q, k_cache, v_cache, cache_len, k_blk, v_blk, out};
+  const char* names[] = {"q", "k_cache", "v_cache", "cache_len", "k_blk", "v_blk", "out"};
+  for (int i = 0; i < 7; ++i) {
+    if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
+    if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
+  }
+  sbd::AttnPlan p = sbd::attn_plan(*desc);
+  p.n_causal = n_causal;
+  const size_t need = sbd::attn_workspace_bytes(p);
+  if (need > 0) {
+    if (!workspace || workspace_bytes < need)
+      return fail(SBD_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
+                  workspace ? workspace_bytes : (size_t)0);
+    if (!aligned16(workspace)) return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+  }
+  return sbd::attn_launch(p, q, k_cache, v_cache, cache_len, k_blk, v_blk, out, workspace, kc_app,
+                          vc_app, (cudaStream_t)stream);
+}
+
 }  // namespace
 
 extern "C" {
@@ -189,25 +215,21 @@ sbd_status sbd_block_attention(const sbd_attn_desc* desc, const void* q, const v
                                const void* v_cache, const int32_t* cache_len, const void* k_blk,
                                const void* v_blk, void* out, void* workspace,
                                size_t workspace_bytes, void* stream) {
-  sbd_status s = check_attn_desc(desc);
-  if (s != SBD_OK) return s;
-  if (desc->batch == 0) return SBD_OK;
-  const void* ptrs[] = {q, k_cache, v_cache, cache_len, k_blk, v_blk, out};
-  const char* names[] = {"q", "k_cache", "v_cache", "cache_len", "k_blk", "v_blk", "out"};
-  for (int i = 0; i < 7; ++i) {
-    if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
-    if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
-  }
-  const sbd::AttnPlan p = sbd::attn_plan(*desc);
-  const size_t need = sbd::attn_workspace_bytes(p);
-  if (need > 0) {
-    if (!workspace || workspace_bytes < need)
-      return fail(SBD_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
-                  workspace ? workspace_bytes : (size_t)0);
-    if (!aligned16(workspace)) return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
-  }
-  return sbd::attn_launch(p, q, k_cache, v_cache, cache_len, k_blk, v_blk, out, workspace,
-                          (cudaStream_t)stream);
+  return attn_call(desc, 0, q, k_cache, v_cache, cache_len, k_blk, v_blk, out, workspace,
+                   workspace_bytes, nullptr, nullptr, stream);
+}
+
+sbd_status sbd_block_attention_causal_prefix(const sbd_attn_desc* desc, int32_t n_causal,
+                                             const void* q, void* k_cache, void* v_cache,
+                                             const int32_t* cache_len, const void* k_blk,
+                                             const void* v_blk, void* out, void* workspace,
+                                             size_t workspace_bytes, void* stream) {
+  if (desc && (n_causal < 0 || n_causal > desc->block_k))
+    return fail(SBD_ERR_INVALID_ARG, "n_causal %d outside [0, block_k = %d]", n_causal,
+                desc->block_k);
+  return attn_call(desc, n_causal, q, k_cache, v_cache, cache_len, k_blk, v_blk, out, workspace,
+                   workspace_bytes, n_causal > 0 ? k_cache : nullptr,
+                   n_causal > 0 ? v_cache : nullptr, stream);
 }
 
 size_t sbd_head_entropy_sample_workspace_size(const sbd_head_desc* desc) {

@@ -28,19 +28,23 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
 // validated by the API layer.
 struct AttnPlan {
   int B, k, Hq, Hkv, G, D, Lmax, M, splits, stages, MT, KG;
+  int n_causal;       // block rows i < n_causal see block keys j <= i only
   float scale_log2;   // softmax scale * log2(e)
   bool bf16;
 };
 size_t attn_workspace_bytes(const AttnPlan& p);
 AttnPlan attn_plan(const sbd_attn_desc& d);
+// kc_app / vc_app: when not NULL (the caches, writable), the keys and values
+// of block rows i < p.n_causal are written at cache position L_b + i.
 sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const void* vc,
                        const int32_t* lens, const void* kb, const void* vb, void* out,
-                       void* ws, cudaStream_t st);
+                       void* ws, void* kc_app, void* vc_app, cudaStream_t st);
 
 size_t attn_tc_smem_bytes(int D);
 sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
                           const void* q, const int32_t* lens, const void* kb, const void* vb,
-                          void* out, float* part_o, float* part_lse, cudaStream_t st);
+                          void* out, float* part_o, float* part_lse, void* kc_app,
+                          void* vc_app, cudaStream_t st);
 
 struct HeadPlan {
   int B, k, H, V, rows_alloc, n_ctas;

@@ -88,6 +88,21 @@ def test_attention_rejects_null_and_misaligned(sbd):
     assert sbd.lib.sbd_block_attention(None, a, a, a, a, a, a, a, None, 0, None) == 1
 
 
+def test_causal_prefix_rejects_bad_arguments(sbd):
+    a = 1 << 20
+    d = _attn_desc(sbd, block_k=32)
+    f = sbd.lib.sbd_block_attention_causal_prefix
+    for nc in (-1, 33):
+        assert f(ctypes.byref(d), nc, a, a, a, a, a, a, a, None, 0, None) == sbd.SBD_ERR_INVALID_ARG
+        assert b"n_causal" in sbd.lib.sbd_last_error()
+    d = _attn_desc(sbd, block_k=33)
+    assert f(ctypes.byref(d), 4, a, a, a, a, a, a, a, None, 0, None) == sbd.SBD_ERR_UNSUPPORTED
+    d = _attn_desc(sbd, head_dim=96)
+    assert f(ctypes.byref(d), 4, a, a, a, a, a, a, a, None, 0, None) == sbd.SBD_ERR_UNSUPPORTED
+    d = _attn_desc(sbd, dtype=sbd.SBD_DTYPE_F32)
+    assert f(ctypes.byref(d), 4, a, None, a, a, a, a, a, None, 0, None) == sbd.SBD_ERR_INVALID_ARG
+
+
 def test_head_rejects_bad_arguments(sbd):
     a = 1 << 20
     d = sbd.HeadDesc(32, 17, 4096, 128256, sbd.SBD_DTYPE_BF16)      # 544 rows > 512
