@@ -681,7 +681,8 @@ def run_sweep(args):
         "per_call_us": {"attention_32_layers": round(attn_ms * 1000, 3),
                         "head": round(head_ms * 1000, 3), "eb_select": round(eb_ms * 1000, 3)},
         "roofline": {
-            "kernel": "block attention, 32 layers (attn_bf16_kernel + split combine)",
+            "kernel": "block attention, 32 layers (attn_tc_kernel, or attn_bf16_kernel at "
+                      "16 packed rows or fewer, + split combine when split)",
             "bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"],
             "peak_source": peak_src, "unit": "GB/s", "frac": round(attn_gbs / peaks["hbm_gbs"], 4),
             "traffic": None, "algorithmic_bytes": int(attn_bytes)},

@@ -584,23 +584,16 @@ attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc,
 
 namespace sbd {
 
+// KV splits per (sequence, KV head): one wave of CTAs, each as long as
+// possible.  A CTA pays a fixed start (tensor memory, barriers, Q, the first
+// loads' latency) and drain; measured on the long-cache workloads, filling
+// further waves with shorter CTAs loses more than the idle SMs of one wave.
 static int choose_splits(int pairs, int n_tiles_max, int sms) {
-  if (pairs >= 2 * sms) return 1;
+  int s = pairs >= sms ? 1 : sms / pairs;
   int max_s = n_tiles_max / 2;
   if (max_s < 1) max_s = 1;
   if (max_s > 32) max_s = 32;
-  int best = 1;
-  double best_eff = 0.0;
-  for (int s = 1; s <= max_s; ++s) {
-    const long long ctas = (long long)pairs * s;
-    const long long waves = (ctas + sms - 1) / sms;
-    const double eff = (double)ctas / (double)(waves * sms);
-    if (eff > best_eff + 0.02) {
-      best_eff = eff;
-      best = s;
-    }
-  }
-  return best;
+  return s < max_s ? s : max_s;
 }
 
 AttnPlan attn_plan(const sbd_attn_desc& d) {
@@ -710,9 +703,11 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.part_o = (float*)ws;
   a.part_lse = p.splits > 1 ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
 
-  // Up to 16 packed rows the mma.sync kernel measures faster (the tcgen05
-  // kernel pads every tile to 128 rows); above, tcgen05.
-  if (SBD_ATTN_TC && p.M > 16) {
+  // Up to 32 packed rows the mma.sync kernel measures faster (the tcgen05
+  // kernel pads every tile to 128 rows, and a TMEM lane quadrant -- 32 rows
+  // -- is read by the warps of one SM sub-partition only, so 32 rows leave
+  // the softmax to one sub-partition); above, tcgen05.
+  if (SBD_ATTN_TC && p.M > 32) {
     s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, kc_app, vc_app,
                        st);
     if (s != SBD_OK) return s;
