@@ -11,16 +11,20 @@
 //   O  += P_j V_j     A = P_j (bf16, shared, K-major), B = V tile (shared,
 //                     MN-major: keys are K, head dims N), fp32 O in TMEM.
 //
-// Warp roles: warp 0 streams K/V tiles with TMA (4-stage ring) and copies
+// Warp roles: warp 0 streams K/V tiles with TMA (6-stage ring) and copies
 // the k block keys/values as the last tile of the last split; warp 1 owns
 // the tensor memory and one thread issues the MMAs, computing S_{j+1} while
-// the softmax of tile j runs; warps 2-5 are the softmax: thread = row, it
-// reads its 64 scores with tcgen05.ld, applies the mask (cache key < L_b,
-// block key < k, or j <= i for a causal block row i < n_causal) and the scale, and writes P_j = 2^(s - m_ref) as bf16 into
-// shared memory.  The reference max m_ref only moves (and O is rescaled in
-// tensor memory) when the running max exceeds it by more than 2^8, which
-// keeps every P entry <= 256; l and O use the same reference, so the result
-// is exact.  The epilogue normalises O by l and writes the output (one split)
+// the softmax of tile j runs; warps 2-9 are the softmax, two per TMEM lane
+// quadrant (and, with 64 packed rows or fewer, each row copied to a second
+// quadrant, so that four warps share a row): a thread reads its share of a
+// row's 64 scores with tcgen05.ld, applies the mask (cache key < L_b,
+// block key < k, or j <= i for a causal block row i < n_causal) and the
+// scale, and writes its part of P_j = 2^(s - m_ref) as bf16 into shared
+// memory.  The warps sharing a row agree on the tile's row maximum through a
+// shared-memory exchange.  The reference max m_ref only moves (and O is
+// rescaled in tensor memory) when the running max exceeds it by more than
+// 2^8, which keeps every P entry <= 256; l and O use the same reference, so
+// the result is exact.  The epilogue normalises O by l and writes the output (one split)
 // or the split partial and its log-sum-exp.
 #include <math.h>
 
@@ -33,12 +37,15 @@ using namespace sbd_dev;
 constexpr int kTileKeys = 64;
 constexpr int kMaxStages = 6;
 constexpr int kRows = 128;                 // MMA M (packed rows, padded)
-constexpr int kThreads = 192;              // producer, MMA, 4 softmax warps
+constexpr int kSoftWarps = 8;              // two per TMEM lane quadrant
+constexpr int kThreads = 64 + 32 * kSoftWarps;   // producer, MMA, softmax warps
 constexpr float kRescaleThreshold = 8.f;   // log2 units
-// Cache tiles are prefetched into L2 this many tiles ahead of the ring, so
-// that the ring's loads see L2 rather than HBM latency.
+// Cache tiles can be prefetched into L2 this many tiles ahead of the ring.
+// Off by default: with one wave of long CTAs the extra requests measured
+// slower (batch 16 x 8192 cache, k = 16: 128 us per layer without, 152 us
+// with 8 tiles ahead).
 #ifndef SBD_ATTN_L2_AHEAD
-#define SBD_ATTN_L2_AHEAD 8
+#define SBD_ATTN_L2_AHEAD 0
 #endif
 
 // ------------------------------------------------------------ tcgen05 PTX
@@ -127,6 +134,16 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
                "r"(v.w)
                : "memory");
 }
+// bf16 bit pattern of the smallest bf16 >= x (x not NaN), and back.
+__device__ __forceinline__ uint16_t bf16_bits_round_up(float x) {
+  const uint32_t u = __float_as_uint(x);
+  const bool neg = (u >> 31) != 0;
+  // positive: round the magnitude up; negative: truncate the magnitude
+  return (uint16_t)((neg ? u : u + 0xFFFFu) >> 16);
+}
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
+  return __uint_as_float((uint32_t)b << 16);
+}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -147,7 +164,13 @@ struct TcArgs {
   float scale_log2;
 };
 
-template <int D>
+// Softmax work split.  R = 1: packed row r lives in TMEM lane r, and the two
+// warps of its lane quadrant take 32 of the tile's 64 columns each.  R = 2
+// (M <= 64): rows are also copied to lanes 64 + r (the MMA pads to 128 rows
+// anyway), so four warps on all four SM sub-partitions share a row, 16
+// columns each.  The warps sharing a row exchange their partial maxima
+// through shared memory at a named barrier and take identical decisions.
+template <int D, int R>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                const __grid_constant__ CUtensorMap tmap_v, const TcArgs a) {
@@ -168,6 +191,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
   __shared__ __align__(8) uint64_t q_ready, tail_bar;
   __shared__ uint32_t tmem_base_sh;
+  // Exchange buffer of the softmax warps: partial row maxima as bf16 rounded
+  // up ([tile parity][warp][lane]), then, at the end, fp32 partial row sums
+  // ([warp][lane]).  1 KB: the ring and Q take the rest of the 227 KB.
+  __shared__ __align__(16) uint32_t red_buf[kSoftWarps * 32];
+  uint16_t* red_max = reinterpret_cast<uint16_t*>(red_buf);
+  float* red_l = reinterpret_cast<float*>(red_buf);
 
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   const uint32_t q_s = sbase;                              // kSub x 16 KB
@@ -184,11 +213,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 4);      // one arrival per softmax warp
-      mbar_init(&p_full[i], 4);
+      mbar_init(&s_free[i], kSoftWarps);      // one arrival per softmax warp
+      mbar_init(&p_full[i], kSoftWarps);
       mbar_init(&pv_done[i], 1);
     }
-    mbar_init(&q_ready, 4);
+    mbar_init(&q_ready, kSoftWarps);
     mbar_init(&tail_bar, 1);
     fence_mbar_init();
   }
@@ -330,6 +359,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         return true;
       };
       if (ok) ok = wait_issue_s(0);
+      // (Issuing PV_j ahead of S_{j+1} when P_j is ready first measured
+      // slower: the next tile's softmax then waits longer for its scores.)
       for (int j = 0; j < n && ok; ++j) {
         if (j + 1 < n && !wait_issue_s(j + 1)) break;
         if (!mbar_wait(&p_full[j & 1], (j >> 1) & 1, a.err)) break;
@@ -339,25 +370,31 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
   } else {
     // ------------------------------------------------ softmax warps
-    const int quad = warp & 3;                  // TMEM lanes 32*quad .. +31
-    const int row = quad * 32 + lane;           // packed row = TMEM lane
+    constexpr int kCW = kTileKeys / (2 * R);     // columns per warp: 32 or 16
+    constexpr int kRowsPerCopy = kRows / R;
+    constexpr int kGroupThreads = 64 * R;        // the warps that share a row
+    const int sw = warp - 2;                     // 0..7
+    const int quad = warp & 3;                   // TMEM lanes 32*quad .. +31
+    const int sub = sw >> 2;                     // 0 or 1 within the quadrant
+    const int lane_t = quad * 32 + lane;         // TMEM lane
+    const int row = lane_t % kRowsPerCopy;       // packed row
+    const int dup = lane_t / kRowsPerCopy;       // copy of the row (R = 2)
+    const int cbase = kCW * (dup * 2 + sub);     // this warp's columns of a tile
+    const bool owns_o = dup == 0;                // O row `row` lives in this lane
+    const int bar_id = 1 + (R == 1 ? quad : (quad & 1));
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
-    // Q row -> shared (swizzled, K-major); padding rows are zero.
+    // softmax warp index of (quadrant q, sub s)
+    auto sw_of = [](int q, int s_) { return 4 * s_ + ((q - 2) & 3); };
+    // Q row -> shared (swizzled, K-major); each sub-warp copies half a row;
+    // padding rows are zero.
     {
       const __nv_bfloat16* qrow =
           row < a.M ? a.q + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
                     : nullptr;
 #pragma unroll
-      for (int c = 0; c < D / 8; ++c) {
+      for (int c = sub * (D / 16); c < (sub + 1) * (D / 16); ++c) {
         const uint4 v = qrow ? *reinterpret_cast<const uint4*>(qrow + c * 8) : make_uint4(0, 0, 0, 0);
-        st_shared_v4(swz(q_s + (c / 8) * kQBytes, row, c % 8), v);
-      }
-      if (!kPInK && quad * 32 >= a.M) {
-        // rows of these warps are never written: keep their P rows zero
-        for (int c = 0; c < 8; ++c) {
-          st_shared_v4(swz(p_s, row, c), make_uint4(0, 0, 0, 0));
-          st_shared_v4(swz(p_s + kQBytes, row, c), make_uint4(0, 0, 0, 0));
-        }
+        st_shared_v4(swz(q_s + (c / 8) * kQBytes, lane_t, c % 8), v);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -365,59 +402,69 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j < n && ok; ++j) {
+    // Every softmax warp runs all n iterations and meets its group barrier
+    // once per iteration, also after a bounded wait gave up (then it only
+    // keeps the barrier count), so that no named barrier waits forever.
+    for (int j = 0; j < n; ++j) {
       const int t = t_begin + j;
       int valid = t < n_cache_tiles ? min(kTileKeys, len - t * kTileKeys) : a.k;
       // causal rows of the block see the block keys j <= i only
       if (t >= n_cache_tiles && row / a.G < a.n_causal) valid = row / a.G + 1;
-      if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float s[kTileKeys];
-      {
-        uint32_t r0[16], r1[16], r2[16], r3[16];
-        const uint32_t sa = tmem + lane_addr + (uint32_t)((j & 1) * kTileKeys);
-        tc_ld16(sa, r0);
-        tc_ld16(sa + 16, r1);
-        tc_ld16(sa + 32, r2);
-        tc_ld16(sa + 48, r3);
-        tc_wait_ld();
+      if (ok && !mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) ok = false;
+      float s[kCW];
+      float mloc = -INFINITY;
+      if (ok) {
+        tc_fence_after();
+        const uint32_t sa = tmem + lane_addr + (uint32_t)((j & 1) * kTileKeys + cbase);
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          s[e] = __uint_as_float(r0[e]);
-          s[16 + e] = __uint_as_float(r1[e]);
-          s[32 + e] = __uint_as_float(r2[e]);
-          s[48 + e] = __uint_as_float(r3[e]);
+        for (int h = 0; h < kCW / 16; ++h) {
+          uint32_t r[16];
+          tc_ld16(sa + 16 * h, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) s[16 * h + e] = __uint_as_float(r[e]);
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free[j & 1]);
+        // masked keys only exist in the last cache tile and the block tile
+        if (valid < cbase + kCW) {
+#pragma unroll
+          for (int c = 0; c < kCW; ++c)
+            if (cbase + c >= valid) s[c] = -INFINITY;
+        }
+        float mx[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx[e] = s[e];
+#pragma unroll
+        for (int c = 8; c < kCW; c += 8)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[c + e]);
+        mloc = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[j & 1]);
-      // masked keys only exist in the last cache tile and the block tile
-      if (valid < kTileKeys) {
+      // The group agrees on max_w(round_up_bf16(m_w)) >= the row maximum: a
+      // reference at or above the maximum is all the lazy rescale needs (l and
+      // O share it), and every warp of the group takes the same value.
+      red_max[((j & 1) * kSoftWarps + sw) * 32 + lane] = bf16_bits_round_up(mloc);
+      asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
+      if (!ok) continue;
+      float mraw = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < kTileKeys; ++c)
-          if (c >= valid) s[c] = -INFINITY;
-      }
-      float mx[8];
+      for (int d2 = 0; d2 < R; ++d2)
 #pragma unroll
-      for (int e = 0; e < 8; ++e) mx[e] = s[e];
-#pragma unroll
-      for (int c = 8; c < kTileKeys; c += 8)
-#pragma unroll
-        for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], s[c + e]);
-      const float mraw = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        for (int s2 = 0; s2 < 2; ++s2) {
+          const int w2 = sw_of((quad & 1) + 2 * d2 + (R == 1 ? (quad & 2) : 0), s2);
+          mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((j & 1) * kSoftWarps + w2) * 32 + lane]));
+        }
       const float mt = mraw * a.scale_log2;     // the scale is positive
       const bool rescale = m_ref != -INFINITY && mt > m_ref + kRescaleThreshold;
       // The P buffer of this tile is free once PV(j-2) is done; O itself is
       // only touched (rescaled) after PV(j-1).
-      const int wait_j = rescale ? j - 1 : (kPInK ? -1 : j - 2);
+      const int wait_j = (rescale && owns_o) ? j - 1 : (kPInK ? -1 : j - 2);
       if (wait_j >= 0 && !mbar_wait(&pv_done[wait_j & 1], (wait_j >> 1) & 1, a.err)) {
         ok = false;
-        break;
+        continue;
       }
       tc_fence_after();
       if (m_ref == -INFINITY) {
@@ -425,41 +472,42 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       } else if (rescale) {
         const float alpha = exp2f(m_ref - mt);
         l *= alpha;
+        if (owns_o) {
+          // the two sub-warps of the row's own quadrant rescale half of O each
 #pragma unroll
-        for (int c = 0; c < D / 16; ++c) {
-          uint32_t r[16];
-          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
-          tc_wait_ld();
+          for (int c = sub * (D / 32); c < (sub + 1) * (D / 32); ++c) {
+            uint32_t r[16];
+            tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+            tc_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-          tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+            for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+            tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+          }
+          tc_wait_st();
         }
-        tc_wait_st();
         m_ref = mt;
       }
-      // P = 2^(scale * s - m_ref) as bf16 into the tile's P buffer (row =
-      // thread); warps holding only padding rows write zeros.
+      // P = 2^(scale * s - m_ref) as bf16 into this warp's columns of the
+      // tile's P buffer (row `row`).  Rows past M and, with R = 2, rows 64+
+      // of P are never written: their O rows are garbage that is never read.
       const uint32_t pb =
           kPInK ? kv_s + (j % kStages) * kStageBytes : p_s + (j & 1) * kQBytes;
-      if (quad * 32 < a.M) {
+      {
         const float nm = -m_ref;
         float psum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int c = 0; c < kTileKeys / 8; ++c) {
+        for (int c = 0; c < kCW / 8; ++c) {
           float p[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             p[e] = exp2f(fmaf(s[c * 8 + e], a.scale_log2, nm));
             psum[e] += p[e];
           }
-          st_shared_v4(swz(pb, row, c), make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
-                                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7])));
+          st_shared_v4(swz(pb, row, cbase / 8 + c),
+                       make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
+                                  pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7])));
         }
         l += ((psum[0] + psum[1]) + (psum[2] + psum[3])) + ((psum[4] + psum[5]) + (psum[6] + psum[7]));
-      } else if (kPInK) {
-        // the K tile under this P tile is not zero: clear the padding rows
-#pragma unroll
-        for (int c = 0; c < kTileKeys / 8; ++c) st_shared_v4(swz(pb, row, c), make_uint4(0, 0, 0, 0));
       }
       fence_proxy_async_smem();
       tc_fence_before();
@@ -468,16 +516,29 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     grid_dependents_launch();
     // ------------------------------------------------ epilogue
-    if (ok && n > 0 && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err)) {
+    // Row sums over the group, in a fixed order.  The first barrier lets the
+    // group finish reading the last tile's maxima before the buffer is reused.
+    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
+    red_l[sw * 32 + lane] = l;
+    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
+    float lsum = 0.f;
+#pragma unroll
+    for (int d2 = 0; d2 < R; ++d2)
+#pragma unroll
+      for (int s2 = 0; s2 < 2; ++s2)
+        lsum += red_l[sw_of((quad & 1) + 2 * d2 + (R == 1 ? (quad & 2) : 0), s2) * 32 + lane];
+    const bool mine = owns_o && row < a.M;
+    // the two sub-warps of the row's quadrant write half of the D columns each
+    const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
+    if (ok && n > 0 && owns_o && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err)) {
       tc_fence_after();
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      const bool mine = row < a.M;
+      const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
       if (a.splits == 1) {
         __nv_bfloat16* dst =
             mine ? a.out + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
                  : nullptr;
 #pragma unroll
-        for (int c = 0; c < D / 16; ++c) {
+        for (int c = c_lo; c < c_hi; ++c) {
           uint32_t r[16];
           tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
           tc_wait_ld();
@@ -499,7 +560,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
         float* dst = mine ? a.part_o + prow * D : nullptr;
 #pragma unroll
-        for (int c = 0; c < D / 16; ++c) {
+        for (int c = c_lo; c < c_hi; ++c) {
           uint32_t r[16];
           tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
           tc_wait_ld();
@@ -511,13 +572,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                               __uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
           }
         }
-        if (mine) a.part_lse[prow] = l > 0.f ? m_ref + log2f(l) : -INFINITY;
+        if (mine && sub == 0) a.part_lse[prow] = lsum > 0.f ? m_ref + log2f(lsum) : -INFINITY;
       }
-    } else if (n == 0 && a.splits > 1 && row < a.M) {
+    } else if (n == 0 && a.splits > 1 && mine) {
       // an empty split contributes nothing
       const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
-      for (int d = 0; d < D; ++d) a.part_o[prow * D + d] = 0.f;
-      a.part_lse[prow] = -INFINITY;
+      for (int d = c_lo * 16; d < c_hi * 16; ++d) a.part_o[prow * D + d] = 0.f;
+      if (sub == 0) a.part_lse[prow] = -INFINITY;
     }
   }
   tc_fence_before();
@@ -566,7 +627,9 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t smem = attn_tc_smem_bytes(p.D);
-  const void* fn = p.D == 128 ? (const void*)attn_tc_kernel<128> : (const void*)attn_tc_kernel<64>;
+  const bool rep2 = p.M <= kRows / 2;
+  const void* fn = p.D == 128 ? (rep2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>)
+                              : (rep2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>);
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
   CUtensorMap k_map = tk, v_map = tv;
