@@ -381,3 +381,56 @@ def select_step(entropy_bk, confidence_bk, token_bk, masked_bk, block_tokens_bk,
         accepted.append(acc)
         orders.append(order)
     return new_masked, new_bt, n_un, accepted, orders
+
+
+# ------------------------------------------- counter-based Gumbel noise
+
+PHILOX_M0, PHILOX_M1 = 0xD2511F53, 0xCD9E8D57       # round multipliers
+PHILOX_W0, PHILOX_W1 = 0x9E3779B9, 0xBB67AE85       # key schedule increments
+
+
+def philox4x32_10(ctr, key):
+    """Philox4x32 with 10 rounds (Salmon, Moraes, Dror, Shaw, "Parallel random
+    numbers: as easy as 1, 2, 3", SC 2011), vectorised over the leading axis.
+    ctr: uint32 [..., 4]; key: uint32 [..., 2].  Each round multiplies words
+    0 and 2 by the round constants (64-bit products split into high and low
+    halves) and mixes in words 1 and 3 and the key; the key grows by the Weyl
+    increments between rounds.  Returns uint32 [..., 4]."""
+    c = np.array(ctr, dtype=np.uint64) & 0xFFFFFFFF
+    k = np.array(key, dtype=np.uint64) & 0xFFFFFFFF
+    c0, c1, c2, c3 = c[..., 0], c[..., 1], c[..., 2], c[..., 3]
+    k0, k1 = k[..., 0], k[..., 1]
+    for r in range(10):
+        if r > 0:
+            k0 = (k0 + PHILOX_W0) & 0xFFFFFFFF
+            k1 = (k1 + PHILOX_W1) & 0xFFFFFFFF
+        p0 = c0 * np.uint64(PHILOX_M0)            # < 2^64: exact in uint64
+        p1 = c2 * np.uint64(PHILOX_M1)
+        hi0, lo0 = p0 >> np.uint64(32), p0 & np.uint64(0xFFFFFFFF)
+        hi1, lo1 = p1 >> np.uint64(32), p1 & np.uint64(0xFFFFFFFF)
+        c0, c1, c2, c3 = hi1 ^ c1 ^ k0, lo1, hi0 ^ c3 ^ k1, lo0
+    return np.stack([c0, c1, c2, c3], axis=-1).astype(np.uint32)
+
+
+def philox_gumbel(row_ids, vocab: int, seed: int, offset: int = 0):
+    """Gumbel noise of the in-kernel generator, in float64: for block
+    position n (= b * k + i) and vocabulary id v, x is word v mod 4 of
+    Philox4x32-10 with counter (v div 4, n, offset low, offset high) and key
+    (seed low, seed high); u = ((x >> 8) + 1/2) 2^-24 lies strictly inside
+    (0, 1); g = -log(-log u).  Returns (g [len(row_ids), V] float64,
+    x [len(row_ids), V] uint32)."""
+    n = np.asarray(row_ids, dtype=np.uint64)
+    v = np.arange(vocab, dtype=np.uint64)
+    R = n.shape[0]
+    ctr = np.zeros((R, (vocab + 3) // 4, 4), dtype=np.uint64)
+    ctr[..., 0] = np.arange((vocab + 3) // 4, dtype=np.uint64)[None, :]
+    ctr[..., 1] = n[:, None]
+    ctr[..., 2] = offset & 0xFFFFFFFF
+    ctr[..., 3] = (offset >> 32) & 0xFFFFFFFF
+    key = np.zeros((R, (vocab + 3) // 4, 2), dtype=np.uint64)
+    key[..., 0] = seed & 0xFFFFFFFF
+    key[..., 1] = (seed >> 32) & 0xFFFFFFFF
+    words = philox4x32_10(ctr, key).reshape(R, -1)[:, :vocab]   # word v mod 4 of call v div 4
+    assert words.shape[1] == v.shape[0]
+    u = ((words >> 8).astype(np.float64) + 0.5) * 2.0 ** -24
+    return -np.log(-np.log(u)), words
