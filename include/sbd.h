@@ -167,6 +167,33 @@ sbd_status sbd_head_entropy_confidence_sample(const sbd_head_desc* desc, const v
                                               void* stream);
 
 /* ------------------------------------------------------------------------
+ * sbd_head_entropy_sample with counter-based Gumbel noise generated inside
+ * the kernel instead of read from a [B, k, V] buffer (the buffer read is
+ * 4 R V bytes per call).  The noise of block position n = b * k + i and
+ * vocabulary id v is
+ *   x = word (v mod 4) of Philox4x32-10(counter = (v div 4, n, offset_lo,
+ *       offset_hi), key = (seed_lo, seed_hi))
+ *       (Salmon, Moraes, Dror, Shaw, SC 2011; 10 rounds),
+ *   u = ((x >> 9) + 1/2) * 2^-23   (exact in fp32, strictly inside (0, 1)),
+ *   g = -ln(-ln u)                 (fp32, full-precision logarithms),
+ * and token = argmax_v (z_v + tau * g).  A new offset (or seed) per step
+ * gives fresh noise.  Every other argument, the workspace and the errors are
+ * those of sbd_head_entropy_sample; tau = 0 is greedy.
+ * ---------------------------------------------------------------------- */
+sbd_status sbd_head_entropy_sample_philox(const sbd_head_desc* desc, const void* hidden,
+                                          const void* w, const uint8_t* masked, uint64_t seed,
+                                          uint64_t offset, float tau, float* entropy,
+                                          int32_t* token, void* workspace,
+                                          size_t workspace_bytes, void* stream);
+
+/* The same noise written out: out[r, v] = g(row_ids[r], v) for 0 <= v < vocab.
+ *   row_ids [n_rows] int32 (device): block positions n = b * k + i
+ *   out [n_rows, vocab] fp32 (device)
+ * Supported: n_rows <= 65535. */
+sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t vocab,
+                             uint64_t seed, uint64_t offset, float* out, void* stream);
+
+/* ------------------------------------------------------------------------
  * No-allocation variant of sbd_head_entropy_sample.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory -- a host framework that owns the whole device memory pool,

@@ -416,8 +416,8 @@ def philox_gumbel(row_ids, vocab: int, seed: int, offset: int = 0):
     """Gumbel noise of the in-kernel generator, in float64: for block
     position n (= b * k + i) and vocabulary id v, x is word v mod 4 of
     Philox4x32-10 with counter (v div 4, n, offset low, offset high) and key
-    (seed low, seed high); u = ((x >> 8) + 1/2) 2^-24 lies strictly inside
-    (0, 1); g = -log(-log u).  Returns (g [len(row_ids), V] float64,
+    (seed low, seed high); u = ((x >> 9) + 1/2) 2^-23 lies strictly inside
+    (0, 1) and is exact in fp32 (24 significant bits); g = -log(-log u).  Returns (g [len(row_ids), V] float64,
     x [len(row_ids), V] uint32)."""
     n = np.asarray(row_ids, dtype=np.uint64)
     v = np.arange(vocab, dtype=np.uint64)
@@ -432,5 +432,5 @@ def philox_gumbel(row_ids, vocab: int, seed: int, offset: int = 0):
     key[..., 1] = (seed >> 32) & 0xFFFFFFFF
     words = philox4x32_10(ctr, key).reshape(R, -1)[:, :vocab]   # word v mod 4 of call v div 4
     assert words.shape[1] == v.shape[0]
-    u = ((words >> 8).astype(np.float64) + 0.5) * 2.0 ** -24
+    u = ((words >> 9).astype(np.float64) + 0.5) * 2.0 ** -23
     return -np.log(-np.log(u)), words

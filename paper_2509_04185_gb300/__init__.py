@@ -47,6 +47,8 @@ EXPORTS = (
     "sbd_head_entropy_sample",
     "sbd_head_entropy_sample_noalloc",
     "sbd_head_entropy_confidence_sample",
+    "sbd_head_entropy_sample_philox",
+    "sbd_gumbel_philox",
     "sbd_eb_select",
     "sbd_select",
     "sbd_status_string",
@@ -100,6 +102,12 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_head_entropy_confidence_sample.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, vp,
                                                        f32, vp, vp, vp, vp, sz, vp]
     lib.sbd_head_entropy_confidence_sample.restype = ctypes.c_int
+    u64 = ctypes.c_uint64
+    lib.sbd_head_entropy_sample_philox.argtypes = [ctypes.POINTER(HeadDesc), vp, vp, vp, u64, u64,
+                                                   f32, vp, vp, vp, sz, vp]
+    lib.sbd_head_entropy_sample_philox.restype = ctypes.c_int
+    lib.sbd_gumbel_philox.argtypes = [i32, vp, i32, u64, u64, vp, vp]
+    lib.sbd_gumbel_philox.restype = ctypes.c_int
     lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
     lib.sbd_eb_select.restype = ctypes.c_int
     lib.sbd_select.argtypes = [i32, i32, i32, vp, vp, vp, f32, vp, vp, vp, vp]
@@ -282,6 +290,44 @@ def sbd_head_entropy_confidence_sample(hidden, w, masked, gumbel, tau: float, en
         ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked), _ptr(gumbel), float(tau),
         _ptr(entropy), _ptr(confidence), _ptr(token), _ptr(ws), _nbytes(ws), _stream(stream)))
     return entropy, confidence, token
+
+
+def sbd_head_entropy_sample_philox(hidden, w, masked, seed: int, offset: int, tau: float,
+                                   entropy=None, token=None, *, workspace=None, stream=None):
+    """sbd_head_entropy_sample with the Gumbel noise generated in the kernel
+    from Philox4x32-10 (seed, offset) instead of read from a tensor.
+    Returns (entropy [B,k] fp32, token [B,k] int32)."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, entropy=entropy, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    B, k, _ = hidden.shape
+    if entropy is None:
+        entropy = torch.empty((B, k), dtype=torch.float32, device=hidden.device)
+    if token is None:
+        token = torch.empty((B, k), dtype=torch.int32, device=hidden.device)
+    d = head_desc(hidden, w)
+    ws = _workspace(lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(d)), hidden.device,
+                    workspace)
+    _check(lib.sbd_head_entropy_sample_philox(ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked),
+                                              int(seed), int(offset), float(tau), _ptr(entropy),
+                                              _ptr(token), _ptr(ws), _nbytes(ws), _stream(stream)))
+    return entropy, token
+
+
+def sbd_gumbel_philox(row_ids, vocab: int, seed: int, offset: int, out=None, *, stream=None):
+    """The counter-based noise written out: out[r, v] = g(row_ids[r], v),
+    row_ids int32 block positions (b * k + i).  Returns out [n, vocab] fp32."""
+    torch = _torch()
+    _need_cuda(row_ids=row_ids, out=out)
+    if row_ids.dtype != torch.int32:
+        raise TypeError("row_ids must be int32")
+    n = row_ids.numel()
+    if out is None:
+        out = torch.empty((n, vocab), dtype=torch.float32, device=row_ids.device)
+    _check(lib.sbd_gumbel_philox(n, _ptr(row_ids), int(vocab), int(seed), int(offset), _ptr(out),
+                                 _stream(stream)))
+    return out
 
 
 def sbd_head_entropy_sample_noalloc(hidden, w, masked, gumbel, tau: float, entropy, token, *,

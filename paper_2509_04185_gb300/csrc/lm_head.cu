@@ -24,6 +24,7 @@
 //                        confidence max_v p_v = 1 / S.
 #include <math.h>
 
+#include "philox.cuh"
 #include "sbd_internal.cuh"
 
 namespace {
@@ -311,7 +312,8 @@ compact_rows_kernel(const uint8_t* __restrict__ hidden, const uint8_t* __restric
 
 // ------------------------------------------------------------ bf16 tcgen05
 struct HeadArgs {
-  const float* gumbel;
+  const float* gumbel;   // noise rows [B*k, V] (noise from a buffer)
+  uint32_t seed_lo, seed_hi, off_lo, off_hi;   // counter-based noise (kPhilox)
   const int32_t* row_map;
   const int32_t* n_rows;
   float4* part_msTb;     // [gridDim.x][rows_alloc]
@@ -324,6 +326,9 @@ struct HeadArgs {
   float tau;
 };
 
+// kPhilox: the Gumbel noise is generated in the epilogue (philox.cuh)
+// instead of read from a [B*k, V] buffer.
+template <bool kPhilox>
 __global__ void __launch_bounds__(kHeadThreads, SBD_HEAD_CTAS_PER_SM)
 head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                const __grid_constant__ CUtensorMap tmap_h, const HeadArgs a) {
@@ -478,7 +483,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       // ------------------------------------------------ epilogue warps
       const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
       const int sub = (warp - 2) / 4;          // chunks sub, sub + n_sub, ... of 16 columns
-      const bool noisy = a.tau != 0.f && a.gumbel != nullptr;
+      const bool noisy = a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
       for (int tile = blockIdx.x; sub < n_sub && tile < a.n_tiles; tile += gridDim.x, ++local) {
@@ -493,28 +498,60 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const int stride = 16 * n_sub;
         const int c_first = 16 * sub;
         float gq[kGAhead][16];
+        if constexpr (!kPhilox) {
 #pragma unroll
-        for (int d = 0; d < kGAhead; ++d)
+          for (int d = 0; d < kGAhead; ++d)
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int cn = c_first + d * stride + j;
-            gq[d][j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
-          }
+            for (int j = 0; j < 16; ++j) {
+              const int cn = c_first + d * stride + j;
+              gq[d][j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            }
+        }
         if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
         tc_fence_after();
         for (int c0 = c_first; c0 < R; c0 += stride) {
           float g[16];
+          if constexpr (!kPhilox) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) g[j] = gq[0][j];
+            for (int j = 0; j < 16; ++j) g[j] = gq[0][j];
 #pragma unroll
-          for (int d = 0; d + 1 < kGAhead; ++d)
+            for (int d = 0; d + 1 < kGAhead; ++d)
 #pragma unroll
-            for (int j = 0; j < 16; ++j) gq[d][j] = gq[d + 1][j];
+              for (int j = 0; j < 16; ++j) gq[d][j] = gq[d + 1][j];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int cn = c0 + kGAhead * stride + j;
-            gq[kGAhead - 1][j] =
-                (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            for (int j = 0; j < 16; ++j) {
+              const int cn = c0 + kGAhead * stride + j;
+              gq[kGAhead - 1][j] =
+                  (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            }
+          } else if (noisy) {
+            // The four lanes 4q..4q+3 share vocabulary ids 4(v div 4) ..
+            // +3, i.e. one Philox counter per row: each lane computes the
+            // calls of 4 of the chunk's 16 rows, and a 4 x 4 transpose inside
+            // the group gives every lane word v mod 4 of all 16.
+            const uint32_t vq = (uint32_t)v >> 2;
+            const int i4 = lane & 3;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const int rr = c0 + 4 * t + i4;
+              const uint32_t n = rr < R ? (uint32_t)rmap[rr] : 0u;
+              const uint4 x = sbd_philox::philox4x32_10(make_uint4(vq, n, a.off_lo, a.off_hi),
+                                                        a.seed_lo, a.seed_hi);
+              uint32_t b[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+              for (int d = 0; d < 4; ++d) {
+                // send word (i ^ d); receive word i of the call of row 4t + (i ^ d)
+                const uint32_t send = sbd_philox::word_of(x, i4 ^ d);
+                const uint32_t recv = d == 0 ? send : __shfl_xor_sync(0xffffffffu, send, d);
+#pragma unroll
+                for (int jj = 0; jj < 4; ++jj) b[jj] = (jj == (i4 ^ d)) ? recv : b[jj];
+              }
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj) g[4 * t + jj] = sbd_philox::gumbel_of_word(b[jj]);
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) g[j] = 0.f;
           }
           uint32_t r[16];
           tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
@@ -553,11 +590,13 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 // ------------------------------------------------------------ fp32 SIMT
 // One CTA per 128 vocab rows; z by sequential fp32 FMAs over H; the same
 // column statistics as the tensor-core epilogue.
+template <bool kPhilox>
 __global__ void __launch_bounds__(128)
 head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
                 const float* __restrict__ gumbel, const int32_t* __restrict__ row_map,
                 const int32_t* __restrict__ n_rows, float tau, int V, int H, int rows_alloc,
-                float4* __restrict__ part_msTb, int32_t* __restrict__ part_idx) {
+                float4* __restrict__ part_msTb, int32_t* __restrict__ part_idx,
+                uint4 philox_sk) {
   grid_dependency_wait();
   __shared__ float4 sm[4][32];
   __shared__ int si[4][32];
@@ -565,7 +604,7 @@ head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
   const int v = blockIdx.x * 128 + threadIdx.x;
   const bool valid = v < V;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool noisy = tau != 0.f && gumbel != nullptr;
+  const bool noisy = tau != 0.f && (kPhilox || gumbel != nullptr);
   const float* wrow = w + (size_t)(valid ? v : 0) * H;
   for (int r0 = 0; r0 < R; r0 += 32) {
     const int nr = min(32, R - r0);
@@ -574,7 +613,18 @@ head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
       const float* h = hidden_c + (size_t)(r0 + j) * H;
       float z = 0.f;
       for (int c = 0; c < H; ++c) z = fmaf(h[c], wrow[c], z);
-      const float g = (noisy && valid) ? gumbel[(size_t)row_map[r0 + j] * V + v] : 0.f;
+      float g = 0.f;
+      if (noisy && valid) {
+        if constexpr (kPhilox) {
+          // philox_sk = (seed low, seed high, offset low, offset high)
+          const uint4 x = sbd_philox::philox4x32_10(
+              make_uint4((uint32_t)v >> 2, (uint32_t)row_map[r0 + j], philox_sk.z, philox_sk.w),
+              philox_sk.x, philox_sk.y);
+          g = sbd_philox::gumbel_of_word(sbd_philox::word_of(x, v & 3));
+        } else {
+          g = gumbel[(size_t)row_map[r0 + j] * V + v];
+        }
+      }
       const RowStats cs = warp_column_stats(z, valid, g, tau, v);
       if (lane == j) mine = cs;
     }
@@ -722,7 +772,8 @@ size_t head_workspace_bytes(const HeadPlan& p) { return head_ws_layout(p, nullpt
 
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
-                       float* confidence, int32_t* token, void* ws, cudaStream_t st) {
+                       float* confidence, int32_t* token, void* ws, cudaStream_t st,
+                       const PhiloxNoise* philox) {
   const int BK = p.B * p.k;
   if (BK == 0) return SBD_OK;
   HeadWs W = head_ws_layout(p, ws);
@@ -763,6 +814,10 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     }
     HeadArgs a;
     a.gumbel = gumbel;
+    a.seed_lo = philox ? (uint32_t)philox->seed : 0u;
+    a.seed_hi = philox ? (uint32_t)(philox->seed >> 32) : 0u;
+    a.off_lo = philox ? (uint32_t)philox->offset : 0u;
+    a.off_hi = philox ? (uint32_t)(philox->offset >> 32) : 0u;
     a.row_map = W.row_map;
     a.n_rows = W.n_rows;
     a.part_msTb = W.part_msTb;
@@ -779,12 +834,12 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.tmem_cols = cols;
     a.tau = tau;
     const size_t smem = head_smem_bytes(p.rows_alloc);
-    e = cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
+    const void* fn = philox ? (const void*)head_tc_kernel<true> : (const void*)head_tc_kernel<false>;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
     void* args[] = {(void*)&tw, (void*)&th, (void*)&a};
-    s = launch_pdl((const void*)head_tc_kernel, dim3(p.n_ctas), dim3(kHeadThreads), smem, st,
-                   args, "head_tc_kernel launch");
+    s = launch_pdl(fn, dim3(p.n_ctas), dim3(kHeadThreads), smem, st, args,
+                   "head_tc_kernel launch");
     if (s != SBD_OK) return s;
   } else {
     const float* hc = (const float*)W.hidden_c;
@@ -794,11 +849,16 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     int V = p.V, H = p.H, ra = p.rows_alloc;
     float4* pm = W.part_msTb;
     int32_t* pi = W.part_idx;
+    uint4 sk = make_uint4(0u, 0u, 0u, 0u);
+    if (philox)
+      sk = make_uint4((uint32_t)philox->seed, (uint32_t)(philox->seed >> 32),
+                      (uint32_t)philox->offset, (uint32_t)(philox->offset >> 32));
     void* args[] = {(void*)&hc, (void*)&wf, (void*)&gumbel, (void*)&rm, (void*)&nr,
                     (void*)&tau, (void*)&V,  (void*)&H,      (void*)&ra, (void*)&pm,
-                    (void*)&pi};
-    s = launch_pdl((const void*)head_f32_kernel, dim3(p.n_ctas), dim3(128), 0, st, args,
-                   "head_f32_kernel launch");
+                    (void*)&pi, (void*)&sk};
+    const void* fn =
+        philox ? (const void*)head_f32_kernel<true> : (const void*)head_f32_kernel<false>;
+    s = launch_pdl(fn, dim3(p.n_ctas), dim3(128), 0, st, args, "head_f32_kernel launch");
     if (s != SBD_OK) return s;
   }
   {

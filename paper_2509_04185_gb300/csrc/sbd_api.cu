@@ -244,7 +244,7 @@ namespace {
 sbd_status head_call(const sbd_head_desc* desc, const void* hidden, const void* w,
                      const uint8_t* masked, const float* gumbel, float tau, float* entropy,
                      float* confidence, int32_t* token, void* workspace, size_t workspace_bytes,
-                     void* stream) {
+                     void* stream, const sbd::PhiloxNoise* philox = nullptr) {
   sbd_status s = check_head_desc(desc);
   if (s != SBD_OK) return s;
   if (!(isfinite(tau) && tau >= 0.f))
@@ -258,7 +258,7 @@ sbd_status head_call(const sbd_head_desc* desc, const void* hidden, const void* 
   }
   if (confidence && !aligned16(confidence))
     return fail(SBD_ERR_INVALID_ARG, "confidence is not 16-byte aligned");
-  if (tau != 0.f && !gumbel)
+  if (tau != 0.f && !gumbel && !philox)
     return fail(SBD_ERR_INVALID_ARG, "gumbel is NULL but tau != 0");
   if (gumbel && !aligned16(gumbel))
     return fail(SBD_ERR_INVALID_ARG, "gumbel is not 16-byte aligned");
@@ -269,7 +269,7 @@ sbd_status head_call(const sbd_head_desc* desc, const void* hidden, const void* 
                 workspace ? workspace_bytes : (size_t)0);
   if (!aligned16(workspace)) return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
   return sbd::head_launch(p, hidden, w, masked, tau == 0.f ? nullptr : gumbel, tau, entropy,
-                          confidence, token, workspace, (cudaStream_t)stream);
+                          confidence, token, workspace, (cudaStream_t)stream, philox);
 }
 
 sbd_status select_call(int32_t rule, int32_t batch, int32_t block_k, const float* entropy,
@@ -316,6 +316,27 @@ sbd_status sbd_head_entropy_confidence_sample(const sbd_head_desc* desc, const v
   if (!confidence) return fail(SBD_ERR_INVALID_ARG, "confidence is NULL");
   return head_call(desc, hidden, w, masked, gumbel, tau, entropy, confidence, token, workspace,
                    workspace_bytes, stream);
+}
+
+sbd_status sbd_head_entropy_sample_philox(const sbd_head_desc* desc, const void* hidden,
+                                          const void* w, const uint8_t* masked, uint64_t seed,
+                                          uint64_t offset, float tau, float* entropy,
+                                          int32_t* token, void* workspace,
+                                          size_t workspace_bytes, void* stream) {
+  const sbd::PhiloxNoise noise{seed, offset};
+  return head_call(desc, hidden, w, masked, nullptr, tau, entropy, nullptr, token, workspace,
+                   workspace_bytes, stream, &noise);
+}
+
+sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t vocab,
+                             uint64_t seed, uint64_t offset, float* out, void* stream) {
+  if (n_rows < 0 || vocab < 0)
+    return fail(SBD_ERR_INVALID_ARG, "bad sizes: n_rows=%d vocab=%d", n_rows, vocab);
+  if (n_rows > 65535) return fail(SBD_ERR_UNSUPPORTED, "n_rows %d > 65535", n_rows);
+  if (n_rows == 0 || vocab == 0) return SBD_OK;
+  if (!row_ids) return fail(SBD_ERR_INVALID_ARG, "row_ids is NULL");
+  if (!out) return fail(SBD_ERR_INVALID_ARG, "out is NULL");
+  return sbd::gumbel_fill_launch(n_rows, row_ids, vocab, seed, offset, out, (cudaStream_t)stream);
 }
 
 sbd_status sbd_eb_select(int32_t batch, int32_t block_k, const float* entropy,

@@ -52,9 +52,16 @@ struct HeadPlan {
 };
 HeadPlan head_plan(const sbd_head_desc& d);
 size_t head_workspace_bytes(const HeadPlan& p);
+// Counter-based noise in place of a noise buffer (philox.cuh).
+struct PhiloxNoise {
+  uint64_t seed, offset;
+};
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
-                       float* confidence, int32_t* token, void* ws, cudaStream_t st);
+                       float* confidence, int32_t* token, void* ws, cudaStream_t st,
+                       const PhiloxNoise* philox = nullptr);
+sbd_status gumbel_fill_launch(int n_rows, const int32_t* row_ids, int V, uint64_t seed,
+                              uint64_t offset, float* out, cudaStream_t st);
 
 // rule: an sbd_select_rule value (SBD_SELECT_EB_ENTROPY for sbd_eb_select)
 sbd_status select_launch(int rule, int B, int k, const float* entropy, const float* confidence,

@@ -164,6 +164,22 @@ def test_confidence_head_rejects_bad_arguments(sbd):
         sbd.SBD_ERR_UNSUPPORTED
 
 
+def test_philox_calls_reject_bad_arguments(sbd):
+    a = 1 << 20
+    d = sbd.HeadDesc(32, 17, 4096, 128256, sbd.SBD_DTYPE_BF16)      # 544 rows > 512
+    f = sbd.lib.sbd_head_entropy_sample_philox
+    assert f(ctypes.byref(d), a, a, a, 1, 2, 1.0, a, a, a, 1 << 30, None) == sbd.SBD_ERR_UNSUPPORTED
+    d = sbd.HeadDesc(1, 16, 4096, 128256, sbd.SBD_DTYPE_BF16)
+    for tau in (-1.0, float("nan")):
+        assert f(ctypes.byref(d), a, a, a, 1, 2, tau, a, a, a, 1 << 30, None) == \
+            sbd.SBD_ERR_INVALID_ARG
+    g = sbd.lib.sbd_gumbel_philox
+    assert g(-1, a, 10, 0, 0, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert g(70000, a, 10, 0, 0, a, None) == sbd.SBD_ERR_UNSUPPORTED
+    assert g(4, None, 10, 0, 0, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert g(0, None, 10, 0, 0, None, None) == sbd.SBD_OK
+
+
 def test_binding_refuses_cpu_tensors(sbd):
     import torch
     x = torch.zeros(1, 4, 4, 64)

@@ -52,14 +52,16 @@ def test_counter_layout_of_the_noise():
             key = np.array([seed & 0xFFFFFFFF, seed >> 32], dtype=np.uint32)
             word = int(oracle.philox4x32_10(ctr, key)[v % 4])
             assert int(x[r, v]) == word
-            u = ((word >> 8) + 0.5) / 2 ** 24
+            u = ((word >> 9) + 0.5) / 2 ** 23
             assert g[r, v] == pytest.approx(-math.log(-math.log(u)), rel=1e-14, abs=1e-15)
 
 
 def test_uniforms_and_bounds():
     g, x = oracle.philox_gumbel(np.arange(64), 8192, seed=99)
-    u = ((x >> 8).astype(np.float64) + 0.5) * 2.0 ** -24
-    assert u.min() >= 2.0 ** -25 and u.max() <= 1.0 - 2.0 ** -25
+    u = ((x >> 9).astype(np.float64) + 0.5) * 2.0 ** -23
+    assert u.min() >= 2.0 ** -24 and u.max() <= 1.0 - 2.0 ** -24
+    # every u is an fp32 value (24 significant bits), so the kernel's is exact
+    assert np.array_equal(u.astype(np.float32).astype(np.float64), u)
     # chi-square of 256 equal bins over 2^19 uniforms
     counts = np.bincount((x >> 24).ravel(), minlength=256)
     expected = x.size / 256
