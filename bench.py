@@ -159,16 +159,18 @@ def host_inputs(w: gen.Workload, seed: int):
     return d
 
 
-def algorithmic_bytes(w: gen.Workload, d) -> dict:
+def algorithmic_bytes(w: gen.Workload, d, noise: str = "buffer") -> dict:
     """Bytes the method must move per step: the KV cache rows in use, block
-    K/V, Q and O once; W, the masked hidden rows, their Gumbel rows and the
-    outputs once; the EB state.  Logits are never written."""
+    K/V, Q and O once; W, the masked hidden rows, their Gumbel rows (none
+    with in-kernel noise) and the outputs once; the EB state.  Logits are
+    never written."""
     e = 2 if w.dtype == "bf16" else 4
     B, k, Hq, Hkv, D = w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim
     L = int(np.sum(d["cache_len"]))
     R = int(d["masked"].sum())
     attn = (2 * L * Hkv * D + 2 * B * k * Hkv * D + 2 * B * k * Hq * D) * e + B * 4
-    head = (w.vocab * w.hidden + R * w.hidden) * e + R * w.vocab * 4 + B * k * (1 + 8)
+    noise_bytes = R * w.vocab * 4 if noise == "buffer" else 0
+    head = (w.vocab * w.hidden + R * w.hidden) * e + noise_bytes + B * k * (1 + 8)
     eb = B * k * (4 + 4 + 1 + 4 + 1 + 4) + B * 4
     return {"attention": attn * w.n_layers, "head": head, "eb": eb, "R": R}
 
@@ -221,8 +223,14 @@ def run_ours(args):
 
     attn_call = sbd.prepare_block_attention(T["q"], T["k_cache"], T["v_cache"], T["cache_len"],
                                             T["k_blk"], T["v_blk"], out, ws_a, stream=stream)
-    head_call = sbd.prepare_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau,
-                                                ent, tok, ws_h, stream=stream)
+    if args.noise == "philox":
+        # in-kernel counter-based noise: no noise tensor is read
+        head_call = sbd.prepare_head_entropy_sample_philox(T["hidden"], T["w"], masked, args.seed,
+                                                           0, tau, ent, tok, ws_h, stream=stream)
+    else:
+        head_call = sbd.prepare_head_entropy_sample(T["hidden"], T["w"], masked, T["gumbel"], tau,
+                                                    ent, tok, ws_h, stream=stream)
+    step_inputs = ("q", "k_blk", "v_blk", "hidden") + (("gumbel",) if args.noise == "buffer" else ())
     eb_call = sbd.prepare_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
 
     def step(ev=None):
@@ -310,7 +318,7 @@ def run_ours(args):
     e2e = None
     if not args.skip_e2e:
         host = {}
-        for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
+        for k in step_inputs:
             host[k] = torch.empty_like(T[k], device="cpu").pin_memory()
             host[k].copy_(T[k])
         host["masked"] = masked0.cpu().pin_memory()
@@ -324,7 +332,7 @@ def run_ours(args):
 
         def e2e_step():
             with torch.cuda.stream(stream):
-                for k in ("q", "k_blk", "v_blk", "hidden", "gumbel"):
+                for k in step_inputs:
                     T[k].copy_(host[k], non_blocking=True)
                 masked.copy_(host["masked"], non_blocking=True)
                 bt.copy_(host["block_tokens"], non_blocking=True)
@@ -357,7 +365,7 @@ def run_ours(args):
 
     if rank != 0:
         return
-    ab = algorithmic_bytes(w, d)
+    ab = algorithmic_bytes(w, d, args.noise)
     peaks, peak_src = measured_peaks()
     head_bytes = ab["head"]
     achieved = head_bytes / (head_ms * 1e-3) / 1e9
@@ -389,7 +397,7 @@ def run_ours(args):
             "n_q_heads": w.n_q_heads, "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
             "cache_len": w.cache_len if not isinstance(w.cache_len, tuple) else list(w.cache_len),
             "hidden": w.hidden, "vocab": w.vocab, "masked_rows": ab["R"], "gamma": gamma,
-            "tau": tau, "parallelism": f"replicas{world}",
+            "tau": tau, "noise": args.noise, "parallelism": f"replicas{world}",
             "l2": "inputs larger than L2: the 1.05 GB+ LM-head weight is streamed every step",
         },
         "gpu_launches": int(args.steps * launches_per_step(sbd, T, ws_a)),
@@ -587,8 +595,14 @@ def run_sweep(args):
     attn_calls = [sbd.prepare_block_attention(L_["q"], L_["kc"], L_["vc"], lens, L_["kb"], L_["vb"],
                                               outs[i], ws_a, stream=stream)
                   for i, L_ in enumerate(layers)]
-    head_calls = [sbd.prepare_head_entropy_sample(hidden[s_], Wt, masked, gumbel, args.tau, ent, tok,
-                                                  ws_h, stream=stream) for s_ in range(k)]
+    if args.noise == "philox":
+        # in-kernel noise: a fresh counter offset per step of the block
+        head_calls = [sbd.prepare_head_entropy_sample_philox(hidden[s_], Wt, masked, args.seed, s_,
+                                                             args.tau, ent, tok, ws_h, stream=stream)
+                      for s_ in range(k)]
+    else:
+        head_calls = [sbd.prepare_head_entropy_sample(hidden[s_], Wt, masked, gumbel, args.tau, ent,
+                                                      tok, ws_h, stream=stream) for s_ in range(k)]
     eb_call = sbd.prepare_eb_select(ent, tok, args.gamma, masked, bt, n_un, stream=stream)
 
     def block(ev=None):
@@ -661,7 +675,7 @@ def run_sweep(args):
     e = 2
     attn_bytes = NL * (2 * B * L * Hkv * D + 2 * B * k * Hkv * D + 2 * B * k * Hq * D) * e
     # masked rows average over the steps of a block: k rows at the first step
-    head_bytes_first = V * H * e + B * k * H * e + B * k * V * 4
+    head_bytes_first = V * H * e + B * k * H * e + (B * k * V * 4 if args.noise == "buffer" else 0)
     ms_per_step = total_ms / n_steps
     attn_gbs = attn_bytes / (attn_ms * 1e-3) / 1e9
     line = {
@@ -672,6 +686,7 @@ def run_sweep(args):
         "data": "synthetic (PyTorch seeded device generator; random-init LM head)",
         "config": {"workload": args.workload, "batch": B, "block_k": k, "layers": NL,
                    "cache_len": L, "hidden": H, "vocab": V, "gamma": args.gamma, "tau": args.tau,
+                   "noise": args.noise,
                    "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2: 17 GB of KV caches per step"},
         "steps_per_block": round(n_steps / n_blocks, 3),
@@ -705,6 +720,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--gamma", type=float, default=0.1)
     ap.add_argument("--tau", type=float, default=1.0)
+    ap.add_argument("--noise", choices=["buffer", "philox"], default="buffer",
+                    help="Gumbel noise read from a tensor, or generated in the LM-head kernel")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time eager launches, no CUDA graph")

@@ -431,6 +431,23 @@ def prepare_head_entropy_sample(hidden, w, masked, gumbel, tau: float, entropy, 
                     (d, hidden, w, masked, gumbel, entropy, token, ws))
 
 
+def prepare_head_entropy_sample_philox(hidden, w, masked, seed: int, offset: int, tau: float,
+                                       entropy, token, workspace=None, *,
+                                       stream=None) -> Prepared:
+    """sbd_head_entropy_sample_philox bound to fixed tensors (see Prepared)."""
+    torch = _torch()
+    _need_cuda(hidden=hidden, w=w, masked=masked, entropy=entropy, token=token)
+    if masked.dtype != torch.uint8:
+        raise TypeError("masked must be uint8")
+    d = head_desc(hidden, w)
+    ws = _workspace(lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(d)), hidden.device,
+                    workspace)
+    args = (ctypes.byref(d), _ptr(hidden), _ptr(w), _ptr(masked), int(seed), int(offset),
+            float(tau), _ptr(entropy), _ptr(token), _ptr(ws), _nbytes(ws), _stream(stream))
+    return Prepared(lib.sbd_head_entropy_sample_philox, args,
+                    (d, hidden, w, masked, entropy, token, ws))
+
+
 def prepare_eb_select(entropy, token, gamma: float, masked, block_tokens, n_unmasked, *,
                       stream=None) -> Prepared:
     """sbd_eb_select bound to fixed tensors (see Prepared)."""
