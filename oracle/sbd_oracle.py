@@ -434,3 +434,65 @@ def philox_gumbel(row_ids, vocab: int, seed: int, offset: int = 0):
     assert words.shape[1] == v.shape[0]
     u = ((words >> 9).astype(np.float64) + 0.5) * 2.0 ** -23
     return -np.log(-np.log(u)), words
+
+
+# ------------------------------------------------- theoretical timing model
+
+# Constants of the paper's roofline analysis (Sec. "Timing analysis"): an
+# H100 with FP8 weights and KV (1 byte per element), BF16 attention, and an
+# 8B transformer with 32 query heads of 128 and 8 KV heads.
+ROOFLINE_H100 = dict(bytes_per_el=1, peak_flops=1978e12, peak_flops_attention=989e12,
+                     bandwidth=3.35 * 1024 ** 4, hidden=4096, ffn=4 * 4096, n_heads=32,
+                     head_dim=128, n_kv_heads=8, kv_bytes=1)
+
+
+def roofline_gemm(m: int, n: int, k: int, c=ROOFLINE_H100):
+    """Roofline time of C = A B with A [m, k], B [k, n]: the larger of
+    (m k + k n + m n) elements moved at the bandwidth and 2 m n k flops at
+    the peak.  Returns (seconds, flops)."""
+    io = (m * k + n * k + m * n) * c["bytes_per_el"]
+    flops = 2.0 * m * n * k
+    return max(io / c["bandwidth"], flops / c["peak_flops"]), flops
+
+
+def roofline_attention(block: int, kv_len: int, batch: int, c=ROOFLINE_H100) -> float:
+    """One fused attention kernel: Q, the K and V of the cache, and the
+    output move once; QK^T and PV are the two contractions over the cache
+    length at the attention peak."""
+    tokens = block * batch
+    width = c["n_heads"] * c["head_dim"]
+    q = tokens * width * c["bytes_per_el"]
+    kv = 2 * batch * kv_len * c["n_kv_heads"] * c["head_dim"] * c["kv_bytes"]
+    o = tokens * width * c["bytes_per_el"]
+    flops = 2 * roofline_gemm(tokens, kv_len, width, c)[1]
+    return max((q + kv + o) / c["bandwidth"], flops / c["peak_flops_attention"])
+
+
+def roofline_linear(block: int, batch: int, c=ROOFLINE_H100) -> float:
+    """The layer's GEMMs with the shapes of the paper's analysis, as printed:
+    the FFN up- and down-projections contract over hidden * ffn, and the K and
+    V projections have width n_heads * n_kv_heads (the reading this build
+    takes of the printed model, which reproduces its tables)."""
+    t, h, f = block * batch, c["hidden"], c["ffn"]
+    nh, hd, nkv = c["n_heads"], c["head_dim"], c["n_kv_heads"]
+    shapes = [(t, h, h * f), (t, h * f, h), (t, h, nh * hd), (t, h, nh * nkv), (t, h, nh * nkv),
+              (t, nh * hd, h)]
+    return sum(roofline_gemm(m, n, k, c)[0] for (m, n, k) in shapes)
+
+
+def roofline_forward(block: int, kv_len: int, batch: int, c=ROOFLINE_H100) -> float:
+    """Forward time of one layer for a block of `block` tokens per sequence:
+    attention plus the linear layers (the layer count cancels in ratios)."""
+    return roofline_attention(block, kv_len, batch, c) + roofline_linear(block, batch, c)
+
+
+def block_slowdown(block: int, kv_len: int, batch: int, c=ROOFLINE_H100) -> float:
+    """time(block) / time(1): the cost of a block forward over an NTP one."""
+    return roofline_forward(block, kv_len, batch, c) / roofline_forward(1, kv_len, batch, c)
+
+
+def sbd_speedup(k: int, l: int, time_fn) -> float:
+    """Wall-clock speedup of SBD over NTP for a block of k tokens decoded in
+    l forwards: k time(1) / (time(2k) + (l - 1) time(k)) -- the first forward
+    of a block also carries the previous block's k tokens (2k rows)."""
+    return k * time_fn(1) / (time_fn(2 * k) + (l - 1) * time_fn(k))

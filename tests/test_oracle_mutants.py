@@ -321,3 +321,34 @@ def test_causal_prefix_mutants_are_caught(monkeypatch, mutant):
     pins = [(TA.test_causal_prefix_rows_equal_explicit_mask, (4, 2, 5)),
             (TA.test_all_causal_block_is_torch_causal_prefill, ())]
     assert all(_fails(fn, *args) for fn, args in pins)
+
+
+# ------------------------------------------------------- timing model
+from tests import test_oracle_roofline as TR   # noqa: E402
+
+
+def _speedup_no_first_forward(k, l, time_fn):
+    return k * time_fn(1) / (l * time_fn(k))                   # first forward of k rows, not 2k
+
+
+def _attention_one_contraction(block, kv_len, batch, c=so.ROOFLINE_H100):
+    tokens = block * batch
+    width = c["n_heads"] * c["head_dim"]
+    mem = (2 * tokens * width * c["bytes_per_el"]
+           + 2 * batch * kv_len * c["n_kv_heads"] * c["head_dim"] * c["kv_bytes"])
+    flops = so.roofline_gemm(tokens, kv_len, width, c)[1]      # PV dropped
+    return max(mem / c["bandwidth"], flops / c["peak_flops_attention"])
+
+
+def _linear_corrected_shapes(block, batch, c=so.ROOFLINE_H100):
+    t, h, f = block * batch, c["hidden"], c["ffn"]
+    shapes = [(t, f, h), (t, h, f), (t, h, h), (t, 1024, h), (t, 1024, h), (t, h, h)]
+    return sum(so.roofline_gemm(m, n, k, c)[0] for (m, n, k) in shapes)
+
+
+@pytest.mark.parametrize("name,mutant", [("sbd_speedup", _speedup_no_first_forward),
+                                         ("roofline_attention", _attention_one_contraction),
+                                         ("roofline_linear", _linear_corrected_shapes)])
+def test_timing_model_mutants_are_caught(monkeypatch, name, mutant):
+    _patch(monkeypatch, name, mutant)
+    assert _fails(TR.test_every_printed_cell)
