@@ -411,6 +411,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       // causal rows of the block see the block keys j <= i only
       if (t >= n_cache_tiles && row / a.G < a.n_causal) valid = row / a.G + 1;
       if (ok && !mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) ok = false;
+      // tcgen05.ld/st are warp-collective: the warp goes on only as a whole
+      ok = __all_sync(0xffffffffu, ok);
       float s[kCW];
       float mloc = -INFINITY;
       if (ok) {
@@ -458,34 +460,38 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((j & 1) * kSoftWarps + w2) * 32 + lane]));
         }
       const float mt = mraw * a.scale_log2;     // the scale is positive
+      // Each row decides for itself; the TMEM rescale of O is warp-collective,
+      // so a warp rescales when any of its rows does (alpha = 1 for the rest).
       const bool rescale = m_ref != -INFINITY && mt > m_ref + kRescaleThreshold;
+      const bool warp_rescale = __any_sync(0xffffffffu, rescale);
       // The P buffer of this tile is free once PV(j-2) is done; O itself is
       // only touched (rescaled) after PV(j-1).
-      const int wait_j = (rescale && owns_o) ? j - 1 : (kPInK ? -1 : j - 2);
-      if (wait_j >= 0 && !mbar_wait(&pv_done[wait_j & 1], (wait_j >> 1) & 1, a.err)) {
+      const int wait_j = (warp_rescale && owns_o) ? j - 1 : (kPInK ? -1 : j - 2);
+      bool waited = wait_j < 0 || mbar_wait(&pv_done[wait_j & 1], (wait_j >> 1) & 1, a.err);
+      if (!__all_sync(0xffffffffu, waited)) {
         ok = false;
         continue;
       }
       tc_fence_after();
+      const float alpha = rescale ? exp2f(m_ref - mt) : 1.f;
       if (m_ref == -INFINITY) {
         m_ref = mt;
       } else if (rescale) {
-        const float alpha = exp2f(m_ref - mt);
         l *= alpha;
-        if (owns_o) {
-          // the two sub-warps of the row's own quadrant rescale half of O each
-#pragma unroll
-          for (int c = sub * (D / 32); c < (sub + 1) * (D / 32); ++c) {
-            uint32_t r[16];
-            tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
-            tc_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-            tc_st16(tmem + lane_addr + kOCol + c * 16, r);
-          }
-          tc_wait_st();
-        }
         m_ref = mt;
+      }
+      if (warp_rescale && owns_o) {
+        // the two sub-warps of the rows' own quadrant rescale half of O each
+#pragma unroll
+        for (int c = sub * (D / 32); c < (sub + 1) * (D / 32); ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+        }
+        tc_wait_st();
       }
       // P = 2^(scale * s - m_ref) as bf16 into this warp's columns of the
       // tile's P buffer (row `row`).  Rows past M and, with R = 2, rows 64+
@@ -530,7 +536,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const bool mine = owns_o && row < a.M;
     // the two sub-warps of the row's quadrant write half of the D columns each
     const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
-    if (ok && n > 0 && owns_o && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err)) {
+    bool final_ok = ok && n > 0 && owns_o && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err);
+    final_ok = __all_sync(0xffffffffu, final_ok);   // the reads below are warp-collective
+    if (final_ok) {
       tc_fence_after();
       const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
       if (a.splits == 1) {

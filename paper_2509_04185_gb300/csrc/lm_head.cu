@@ -507,7 +507,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
               gq[d][j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
             }
         }
-        if (!mbar_wait(&tmem_full[acc], use & 1, a.err)) break;
+        // the tcgen05.ld below is warp-collective: the warp goes on as a whole
+        if (!__all_sync(0xffffffffu, mbar_wait(&tmem_full[acc], use & 1, a.err))) break;
         tc_fence_after();
         for (int c0 = c_first; c0 < R; c0 += stride) {
           float g[16];

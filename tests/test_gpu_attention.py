@@ -130,3 +130,34 @@ def test_repeated_calls_leave_no_device_error(sbd, k, L, splits):
     torch.cuda.synchronize()
     assert sbd.sbd_device_error() == 0
     assert torch.equal(out0, ref)
+
+
+@pytest.mark.parametrize("G,k,splits", [(4, 16, 0), (4, 16, 3), (4, 32, 0), (4, 32, 2), (4, 8, 0),
+                                        (1, 16, 1)])
+def test_growing_scores_take_the_rescale_path(sbd, G, k, splits):
+    """Scores that grow along the cache (keys scaled up to 7x toward the end,
+    queries 4x): every row's running maximum jumps by more than the lazy
+    rescale threshold many times, at different tiles for different rows of a
+    warp, so the O rescale runs and must stay exact."""
+    import torch
+    Hkv = 2
+    w = gen.shrink(BF16, batch=2, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv,
+                   cache_len=(900, 1500))
+    d = dict(gen.attention_inputs(w, seed=G * 13 + k, poison_tail=False))
+    q = gen.bf16_bits_to_f32(d["q"]) * 4.0
+    kc = gen.bf16_bits_to_f32(d["k_cache"])
+    ramp = (1.0 + 6.0 * np.arange(kc.shape[1]) / kc.shape[1]).astype(np.float32)
+    kc = kc * ramp[None, :, None, None]
+    d["q"] = gen.f32_to_bf16_bits(q)
+    d["k_cache"] = gen.f32_to_bf16_bits(kc)
+    t = {x: to_dev(d[x], "bf16") for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    lens = torch.from_numpy(d["cache_len"]).cuda()
+    out = sbd.sbd_block_attention(t["q"], t["k_cache"], t["v_cache"], lens, t["k_blk"],
+                                  t["v_blk"], num_splits=splits)
+    got = out.float().cpu().numpy()
+    f = {x: oracle.widen(d[x], "bf16") for x in ("q", "k_cache", "v_cache", "k_blk", "v_blk")}
+    ref = oracle.block_attention(f["q"], f["k_cache"], f["v_cache"], d["cache_len"], f["k_blk"],
+                                 f["v_blk"])
+    assert np.isfinite(got).all()
+    assert float(np.abs(got - ref).max()) <= BF16_ATTN_TOL
+    assert sbd.sbd_device_error() == 0
