@@ -249,6 +249,7 @@ def run_ours(args):
             if ev is not None:
                 ev[3].record(stream)
 
+    torch.cuda.synchronize(dev)        # inputs were made on the default stream
     sampler = ClockSampler(local_rank) if rank == 0 else None
     if sampler:
         sampler.start()
@@ -708,6 +709,192 @@ def run_sweep(args):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------- measured speedup tables
+
+SPEEDUP_BATCHES = (1, 4, 16)
+SPEEDUP_KV_LENS = (1024, 8192, 32768)
+SPEEDUP_KS = (4, 8, 16)
+SPEEDUP_NFE = (2, 4)
+
+
+def run_speedup_tables(args):
+    """GB300 wall-clock counterpart of the paper's theoretical speedup tables
+    (Sec. "Timing analysis"): time(n) of a full forward of a Llama-3.1-8B-
+    shaped model (32 layers, 32/8 heads of 128, hidden 4096, MLP 14336, vocab
+    128256, bf16) for a block of n tokens per sequence, measured for n = 1
+    (NTP), k, and 2k (the first forward of a block, which also carries the
+    previous block's k tokens), then
+        slowdown(n)    = time(n) / time(1),
+        speedup(l, k)  = k time(1) / (time(2k) + (l - 1) time(k)),  l = k / NFE.
+    Per layer (pre-norm, RMSNorm without gain): the fused QKV projection,
+    block attention (sbd_block_attention, or sbd_block_attention_causal_prefix
+    with the first k rows causal for 2k), the output projection and the
+    SiLU-gated MLP; then the final norm and the LM head with entropy and
+    Gumbel-max sample (sbd_head_entropy_sample) over the B n rows.
+    The projections are plain bf16 GEMMs (cuBLAS through torch.matmul): the
+    model's linear layers, outside the SBD step.  Every layer has its own
+    weights and KV cache, so nothing stays in L2 between layers; each forward
+    is one CUDA graph, timed with CUDA events over `--steps` replays."""
+    import torch
+
+    import paper_2509_04185_gb300 as sbd
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    NL, H, F, V, Hq, Hkv, D = 32, 4096, 14336, 128256, 32, 8, 128
+    g = torch.Generator(device=dev)
+    g.manual_seed(args.seed * 7919 + 3)
+
+    def randn(*shape, std=1.0):
+        return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32) * std).bfloat16()
+
+    w_std = 0.02
+    layers_w = [dict(qkv=randn((Hq + 2 * Hkv) * D, H, std=w_std), o=randn(H, Hq * D, std=w_std),
+                     gu=randn(2 * F, H, std=w_std), down=randn(H, F, std=w_std)) for _ in range(NL)]
+    w_head = randn(V, H, std=w_std)
+    stream = torch.cuda.Stream(dev)
+    max_n = 2 * max(SPEEDUP_KS)
+    results = []
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    for B in SPEEDUP_BATCHES:
+        for L in SPEEDUP_KV_LENS:
+            if B * max_n > 512:
+                continue
+            Lmax = L + max_n
+            caches = [(randn(B, Lmax, Hkv, D), randn(B, Lmax, Hkv, D)) for _ in range(NL)]
+            print(f"speedup tables: batch {B} kv {L}: caches ready", file=sys.stderr, flush=True)
+            lens = torch.full((B,), L, dtype=torch.int32, device=dev)
+            # (block rows, causal prefix rows): NTP, the block steps, and the
+            # first forward of each block size
+            forwards = [(1, 0)] + [(k, 0) for k in SPEEDUP_KS] + [(2 * k, k) for k in SPEEDUP_KS]
+            times = {}
+            for n, n_causal in forwards:
+                T = B * n
+                x0 = randn(T, H)
+                attn_out = torch.empty(B, n, Hq, D, dtype=torch.bfloat16, device=dev)
+                ad = sbd.AttnDesc(B, n, Hq, Hkv, D, Lmax, sbd.SBD_DTYPE_BF16, 0.0, 0)
+                import ctypes
+                ws_a = torch.empty(max(1, sbd.lib.sbd_block_attention_workspace_size(ctypes.byref(ad))),
+                                   dtype=torch.uint8, device=dev)
+                hid = torch.empty(B, n, H, dtype=torch.bfloat16, device=dev)
+                masked = torch.ones(B, n, dtype=torch.uint8, device=dev)
+                gum = torch.rand(B, n, V, generator=g, device=dev)
+                ent = torch.empty(B, n, device=dev)
+                tok = torch.empty(B, n, dtype=torch.int32, device=dev)
+                hd = sbd.HeadDesc(B, n, H, V, sbd.SBD_DTYPE_BF16)
+                ws_h = torch.empty(sbd.lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(hd)),
+                                   dtype=torch.uint8, device=dev)
+                qkv_buf = torch.empty(T, (Hq + 2 * Hkv) * D, dtype=torch.bfloat16, device=dev)
+                q_v = qkv_buf[:, :Hq * D].view(B, n, Hq, D)
+                k_v = qkv_buf[:, Hq * D:(Hq + Hkv) * D]
+                v_v = qkv_buf[:, (Hq + Hkv) * D:]
+                kb = torch.empty(B, n, Hkv, D, dtype=torch.bfloat16, device=dev)
+                vb = torch.empty(B, n, Hkv, D, dtype=torch.bfloat16, device=dev)
+                qc = torch.empty(B, n, Hq, D, dtype=torch.bfloat16, device=dev)
+                calls = []
+                for li in range(NL):
+                    kc, vc = caches[li]
+                    if n_causal:
+                        calls.append(lambda kc=kc, vc=vc: sbd.sbd_block_attention_causal_prefix(
+                            qc, kc, vc, lens, kb, vb, n_causal, out=attn_out, workspace=ws_a,
+                            stream=stream))
+                    else:
+                        calls.append(lambda kc=kc, vc=vc: sbd.sbd_block_attention(
+                            qc, kc, vc, lens, kb, vb, out=attn_out, workspace=ws_a, stream=stream))
+
+                def rms(x):
+                    xf = x.float()
+                    return (xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + 1e-5)).bfloat16()
+
+                def forward():
+                    with torch.cuda.stream(stream):
+                        x = x0
+                        for li in range(NL):
+                            Wl = layers_w[li]
+                            torch.matmul(rms(x), Wl["qkv"].t(), out=qkv_buf)
+                            qc.copy_(q_v)                          # contiguous per-call layouts
+                            kb.copy_(k_v.view(B, n, Hkv, D))
+                            vb.copy_(v_v.view(B, n, Hkv, D))
+                            calls[li]()
+                            o = torch.matmul(attn_out.view(T, Hq * D), Wl["o"].t())
+                            x = x + o
+                            gu = torch.matmul(rms(x), Wl["gu"].t())
+                            act = torch.nn.functional.silu(gu[:, :F]) * gu[:, F:]
+                            x = x + torch.matmul(act, Wl["down"].t())
+                        hid.copy_(rms(x).view(B, n, H))
+                        sbd.sbd_head_entropy_sample(hid, w_head, masked, gum, 1.0, ent, tok,
+                                                    workspace=ws_h, stream=stream)
+
+                # the inputs above were made on the default stream
+                torch.cuda.synchronize(dev)
+                for _ in range(3):
+                    forward()
+                torch.cuda.synchronize(dev)
+                graph = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph, stream=stream):
+                    forward()
+                for _ in range(max(3, args.warmup)):
+                    graph.replay()
+                torch.cuda.synchronize(dev)
+                reps = max(5, min(args.steps, 50))
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                with torch.cuda.stream(stream):
+                    for _ in range(reps):
+                        graph.replay()
+                e1.record(stream)
+                torch.cuda.synchronize(dev)
+                times[(n, n_causal)] = e0.elapsed_time(e1) / reps
+                if not bool(torch.isfinite(ent).all()):
+                    raise RuntimeError(f"non-finite entropy at batch {B} kv {L} block {n}")
+                del graph
+                print(f"speedup tables: batch {B} kv {L} block {n} (causal {n_causal}): "
+                      f"{times[(n, n_causal)]:.3f} ms", file=sys.stderr, flush=True)
+            code = sbd.sbd_device_error()
+            if code != 0:
+                raise RuntimeError(f"device error word {code} at batch {B} kv {L}")
+            t1 = times[(1, 0)]
+            name = lambda n, c: f"{n}" if c == 0 else f"{n}_first"
+            row = {"batch": B, "kv_len": L,
+                   "ms_per_forward": {name(n, c): round(t, 4) for (n, c), t in times.items()},
+                   "slowdown": {name(n, c): round(t / t1, 4) for (n, c), t in times.items()},
+                   "speedup": {}}
+            for k in SPEEDUP_KS:
+                for nfe in SPEEDUP_NFE:
+                    l = k // nfe
+                    if l < 1:
+                        continue
+                    row["speedup"][f"k{k}_nfe{nfe}"] = round(
+                        k * t1 / (times[(2 * k, k)] + (l - 1) * times[(k, 0)]), 4)
+            results.append(row)
+            del caches
+            torch.cuda.empty_cache()
+    clocks = sampler.stop() if sampler else None
+    if rank != 0:
+        return
+    ref = next(r for r in results if r["batch"] == 1 and r["kv_len"] == 8192)
+    line = {
+        "metric": "measured wall-clock speedup of block decoding over NTP (k=16, NFE speedup 4, "
+                  "batch 1, KV 8192)",
+        "value": ref["speedup"]["k16_nfe4"], "unit": "x", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (PyTorch seeded device generator; random-init 8B-shaped weights)",
+        "config": {"workload": "speedup_tables", "model": "Llama-3.1-8B shapes, 32 layers",
+                   "batches": list(SPEEDUP_BATCHES), "kv_lens": list(SPEEDUP_KV_LENS),
+                   "block_sizes": list(SPEEDUP_KS), "nfe_speedups": list(SPEEDUP_NFE),
+                   "linear_layers": "cuBLAS bf16 GEMMs (torch.matmul)",
+                   "attention_and_head": "libsbd kernels"},
+        "clocks": clocks,
+        "tables": results,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -716,7 +903,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b_k16",
                     choices=["llama8b_k16", "ragged_b32_k8", "qwen8b_long_k16", "tiny_f32",
-                             "sweep32_k4", "sweep32_k8", "sweep32_k16", "sweep32_k32"])
+                             "sweep32_k4", "sweep32_k8", "sweep32_k16", "sweep32_k32",
+                             "speedup_tables"])
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--gamma", type=float, default=0.1)
     ap.add_argument("--tau", type=float, default=1.0)
@@ -732,6 +920,8 @@ def main():
         run_reference(args)
     elif args.workload.startswith("sweep32"):
         run_sweep(args)
+    elif args.workload == "speedup_tables":
+        run_speedup_tables(args)
     else:
         run_ours(args)
 
