@@ -4,28 +4,37 @@
 // Same partition as the mma.sync kernel -- one CTA per (KV split, KV head,
 // sequence), the G query heads of a KV head packed with the k block rows
 // into one row tile (row r = i*G + g, padded to 128) -- but both products run
-// on tcgen05 with their accumulators in tensor memory:
+// on tcgen05 with their accumulators in tensor memory.  Keys stream in tiles
+// of 64 (one TMA stage each) and the products run on pairs of tiles:
 //
-//   S_j = Q K_j^T     A = Q (shared, K-major), B = K tile (shared, K-major),
-//                     M = 128 rows, N = 64 keys, fp32 in TMEM (2 buffers);
-//   O  += P_j V_j     A = P_j (bf16, shared, K-major), B = V tile (shared,
-//                     MN-major: keys are K, head dims N), fp32 O in TMEM.
+//   S_q = Q K_q^T     A = Q (shared, K-major), B = the pair's K (shared,
+//                     K-major), M = 128 rows, N = 128 keys, fp32 in TMEM
+//                     (2 buffers);
+//   O  += P_q V_q     A = P_q (bf16, shared, K-major), B = the pair's V
+//                     (shared, MN-major: keys are K, head dims N), fp32 O in
+//                     TMEM.
 //
-// Warp roles: warp 0 streams K/V tiles with TMA (6-stage ring) and copies
-// the k block keys/values as the last tile of the last split; warp 1 owns
-// the tensor memory and one thread issues the MMAs, computing S_{j+1} while
-// the softmax of tile j runs; warps 2-9 are the softmax, two per TMEM lane
-// quadrant (and, with 64 packed rows or fewer, each row copied to a second
-// quadrant, so that four warps share a row): a thread reads its share of a
-// row's 64 scores with tcgen05.ld, applies the mask (cache key < L_b,
+// Pairs, not single tiles: an M = 128, K = 16 tcgen05.mma measured about the
+// same time for N = 64, 128 and 256 (~135 cycles), so 64-key score products
+// left the tensor pipe the bottleneck (1300 cycles of MMA per 64 keys; 760
+// with 128-key pairs).  The two tiles of a pair sit back to back in every
+// 128-byte sub-tile of the ring, so that they form one 128-row operand.
+//
+// Warp roles: warp 0 streams K/V tiles with TMA (a ring of 3 pairs) and
+// copies the k block keys/values as the last tile of the last split; warp 1
+// owns the tensor memory and one thread issues the MMAs, computing S_{q+1}
+// while the softmax of pair q runs; warps 2-9 are the softmax, two per TMEM
+// lane quadrant (and, with 64 packed rows or fewer, each row copied to a
+// second quadrant, so that four warps share a row): a thread reads its share
+// of a row's 128 scores with tcgen05.ld, applies the mask (cache key < L_b,
 // block key < k, or j <= i for a causal block row i < n_causal) and the
-// scale, and writes its part of P_j = 2^(s - m_ref) as bf16 into shared
-// memory.  The warps sharing a row agree on the tile's row maximum through a
+// scale, and writes its part of P_q = 2^(s - m_ref) as bf16 into shared
+// memory.  The warps sharing a row agree on the pair's row maximum through a
 // shared-memory exchange.  The reference max m_ref only moves (and O is
 // rescaled in tensor memory) when the running max exceeds it by more than
 // 2^8, which keeps every P entry <= 256; l and O use the same reference, so
-// the result is exact.  The epilogue normalises O by l and writes the output (one split)
-// or the split partial and its log-sum-exp.
+// the result is exact.  The epilogue normalises O by l and writes the output
+// (one split) or the split partial and its log-sum-exp.
 #include <math.h>
 
 #include "sbd_internal.cuh"
@@ -34,8 +43,10 @@ namespace {
 
 using namespace sbd_dev;
 
-constexpr int kTileKeys = 64;
-constexpr int kMaxStages = 6;
+constexpr int kTileKeys = 64;              // keys per TMA stage
+constexpr int kPairKeys = 2 * kTileKeys;   // keys per MMA step (two stages)
+constexpr int kMaxStages = 8;
+constexpr int kMaxPairs = kMaxStages / 2;
 constexpr int kRows = 128;                 // MMA M (packed rows, padded)
 constexpr int kSoftWarps = 8;              // two per TMEM lane quadrant
 constexpr int kThreads = 64 + 32 * kSoftWarps;   // producer, MMA, softmax warps
@@ -164,35 +175,39 @@ struct TcArgs {
   float scale_log2;
 };
 
-// Softmax work split.  R = 1: packed row r lives in TMEM lane r, and the two
-// warps of its lane quadrant take 32 of the tile's 64 columns each.  R = 2
-// (M <= 64): rows are also copied to lanes 64 + r (the MMA pads to 128 rows
-// anyway), so four warps on all four SM sub-partitions share a row, 16
-// columns each.  The warps sharing a row exchange their partial maxima
-// through shared memory at a named barrier and take identical decisions.
+// Softmax work split over the 128 columns of a pair.  R = 1: packed row r
+// lives in TMEM lane r, and the two warps of its lane quadrant take 64 of the
+// pair's 128 columns each (one tile each).  R = 2 (M <= 64): rows are also
+// copied to lanes 64 + r (the MMA pads to 128 rows anyway), so four warps on
+// all four SM sub-partitions share a row, 32 columns each.  The warps sharing
+// a row exchange their partial maxima through shared memory at a named
+// barrier and take identical decisions.
 template <int D, int R>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                const __grid_constant__ CUtensorMap tmap_v, const TcArgs a) {
-  constexpr int kSub = D / 64;                    // 128-B column sub-tiles
-  constexpr int kQBytes = kRows * 128;            // one Q (or P) sub-tile: 16 KB
-  constexpr int kKVSub = kTileKeys * 128;         // one K or V sub-tile: 8 KB
-  constexpr int kStageBytes = 2 * kSub * kKVSub;  // K sub-tiles then V sub-tiles
-  constexpr uint32_t kTmemCols = 256;             // S0 | S1 | O
-  constexpr uint32_t kOCol = 2 * kTileKeys;
-  // With D = 128 the K region of a stage (16 KB) is exactly a P tile, and K is
-  // dead once S_j is computed: P_j is written there, and the ring gets the
-  // shared memory separate P buffers would take.
+  constexpr int kSub = D / 64;                     // 128-B column sub-tiles of a key row
+  constexpr int kQBytes = kRows * 128;             // one Q (or P) sub-tile: 16 KB
+  constexpr int kKVSub = kTileKeys * 128;          // one tile's K or V sub-tile: 8 KB
+  constexpr int kPairSub = 2 * kKVSub;             // a pair's K or V sub-tile: 16 KB
+  constexpr int kPairBytes = 2 * kSub * kPairSub;  // K sub-tiles then V sub-tiles
+  constexpr uint32_t kTmemCols = 512;              // S0 | S1 (128 each) | O
+  constexpr uint32_t kOCol = 2 * kPairKeys;
+  // With D = 128 the K region of a pair (32 KB) is exactly a P block, and K is
+  // dead once S of the pair is computed: P is written there, and the ring gets
+  // the shared memory separate P buffers would take.
   constexpr bool kPInK = D == 128;
-  constexpr int kStages = kPInK ? 6 : 5;
+  constexpr int kPairs = kPInK ? 3 : 4;            // ring depth in pairs
+  constexpr int kStages = 2 * kPairs;              // ring depth in 64-key tiles
+  static_assert(kQBytes == kPairSub, "a P sub-tile fills a pair's K sub-tile");
 
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t kv_full[kMaxStages], kv_empty[kMaxStages];
+  __shared__ __align__(8) uint64_t kv_full[kMaxStages], kv_empty[kMaxPairs];
   __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
   __shared__ __align__(8) uint64_t q_ready, tail_bar;
   __shared__ uint32_t tmem_base_sh;
   // Exchange buffer of the softmax warps: partial row maxima as bf16 rounded
-  // up ([tile parity][warp][lane]), then, at the end, fp32 partial row sums
+  // up ([pair parity][warp][lane]), then, at the end, fp32 partial row sums
   // ([warp][lane]).  1 KB: the ring and Q take the rest of the 227 KB.
   __shared__ __align__(16) uint32_t red_buf[kSoftWarps * 32];
   uint16_t* red_max = reinterpret_cast<uint16_t*>(red_buf);
@@ -200,17 +215,28 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
 
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   const uint32_t q_s = sbase;                              // kSub x 16 KB
-  const uint32_t p_s = q_s + kSub * kQBytes;               // 2 x 16 KB unless kPInK
-  const uint32_t kv_s = p_s + (kPInK ? 0 : 2 * kQBytes);   // kStages x kStageBytes
+  const uint32_t p_s = q_s + kSub * kQBytes;               // 2 x 32 KB unless kPInK
+  const uint32_t kv_s = p_s + (kPInK ? 0 : 4 * kQBytes);   // kPairs x kPairBytes
+  // Tile j of this split lives in pair slot (j / 2) mod kPairs, half j mod 2:
+  // the two tiles of a pair sit back to back in every sub-tile, so that a
+  // pair's keys form one 128-row operand.
+  auto k_chunk = [&](int j, int h) -> uint32_t {
+    return kv_s + ((j >> 1) % kPairs) * kPairBytes + h * kPairSub + (j & 1) * kKVSub;
+  };
+  auto v_chunk = [&](int j, int h) -> uint32_t {
+    return kv_s + ((j >> 1) % kPairs) * kPairBytes + (kSub + h) * kPairSub + (j & 1) * kKVSub;
+  };
+  // P block of pair q: two 16 KB sub-tiles (keys 0-63, 64-127)
+  auto p_block = [&](int q) -> uint32_t {
+    return kPInK ? k_chunk(2 * q, 0) : p_s + (q & 1) * 2 * kQBytes;
+  };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
-    }
+    for (int s = 0; s < kStages; ++s) mbar_init(&kv_full[s], 1);
+    for (int s = 0; s < kPairs; ++s) mbar_init(&kv_empty[s], 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
       mbar_init(&s_free[i], kSoftWarps);      // one arrival per softmax warp
@@ -221,8 +247,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     mbar_init(&tail_bar, 1);
     fence_mbar_init();
   }
-  if (warp == 1) tc_alloc(&tmem_base_sh, kTmemCols);
+  // All 512 tensor-memory columns are taken only after the previous grid is
+  // done, so that no CTA of it can be left waiting for them.
   grid_dependency_wait();
+  if (warp == 1) tc_alloc(&tmem_base_sh, kTmemCols);
 
   int len = a.lens[b];
   if (len < 0 || len > a.Lmax) {
@@ -233,7 +261,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const int n_tiles = n_cache_tiles + 1;
   const int t_begin = (int)((long long)split * n_tiles / a.splits);
   const int t_end = (int)((long long)(split + 1) * n_tiles / a.splits);
-  const int n = t_end - t_begin;
+  const int n = t_end - t_begin;                  // 64-key tiles of this split
+  const int np = (n + 1) / 2;                     // pairs (the last may hold one tile)
 
   tc_fence_before();
   __syncthreads();
@@ -259,22 +288,24 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     for (int j = 0; j < n; ++j) {
       const int t = t_begin + j;
       const int stage = j % kStages;
-      const uint32_t ph = (j / kStages) & 1;
-      if (!mbar_wait(&kv_empty[stage], ph ^ 1, a.err)) break;
-      const uint32_t ks = kv_s + stage * kStageBytes;
-      const uint32_t vs = ks + kSub * kKVSub;
-      uint8_t* kg = smem_raw + (ks - smem_u32(smem_raw));
-      uint8_t* vg = smem_raw + (vs - smem_u32(smem_raw));
+      // a pair slot is reused once the PV product of its previous pair is done
+      if ((j & 1) == 0) {
+        const int q = j >> 1;
+        const bool freed = mbar_wait(&kv_empty[q % kPairs], ((q / kPairs) & 1) ^ 1, a.err);
+        if (!__all_sync(0xffffffffu, freed)) break;
+      }
       if (t < n_cache_tiles) {
         const int valid = min(kTileKeys, len - t * kTileKeys);
         const bool tail = valid < kTileKeys;
         uint64_t* bar = tail ? &tail_bar : &kv_full[stage];
         if (lane == 0) {
           prefetch(t + kStages + SBD_ATTN_L2_AHEAD);
-          mbar_arrive_expect_tx(bar, kStageBytes);
+          mbar_arrive_expect_tx(bar, 2 * kSub * kKVSub);
           for (int h = 0; h < kSub; ++h) {
-            tma_load_4d(kg + h * kKVSub, &tmap_k, bar, 64 * h, hkv, t * kTileKeys, b);
-            tma_load_4d(vg + h * kKVSub, &tmap_v, bar, 64 * h, hkv, t * kTileKeys, b);
+            tma_load_4d(smem_raw + (k_chunk(j, h) - smem_u32(smem_raw)), &tmap_k, bar, 64 * h, hkv,
+                        t * kTileKeys, b);
+            tma_load_4d(smem_raw + (v_chunk(j, h) - smem_u32(smem_raw)), &tmap_v, bar, 64 * h, hkv,
+                        t * kTileKeys, b);
           }
         }
         if (tail) {
@@ -283,7 +314,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           mbar_wait(&tail_bar, 0, a.err);
           for (int c = lane; c < (kTileKeys - valid) * kSub * 8; c += 32) {
             const int row = valid + c / (kSub * 8), h = (c / 8) % kSub, cc = c % 8;
-            st_shared_v4(swz(vs + h * kKVSub, row, cc), make_uint4(0, 0, 0, 0));
+            st_shared_v4(swz(v_chunk(j, h), row, cc), make_uint4(0, 0, 0, 0));
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -306,8 +337,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
               *reinterpret_cast<uint4*>(a.vc_app + dst) = vv;
             }
           }
-          st_shared_v4(swz(ks + (cc / 8) * kKVSub, row, cc % 8), kv);
-          st_shared_v4(swz(vs + (cc / 8) * kKVSub, row, cc % 8), vv);
+          st_shared_v4(swz(k_chunk(j, cc / 8), row, cc % 8), kv);
+          st_shared_v4(swz(v_chunk(j, cc / 8), row, cc % 8), vv);
         }
         if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
           record_error(a.err, SBD_DEVERR_CACHE_LEN);
@@ -319,58 +350,66 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0 && n > 0) {
-      const uint32_t id_s = idesc_bf16(kRows, kTileKeys, false);
       const uint32_t id_o = idesc_bf16(kRows, D, true);
       bool ok = mbar_wait(&q_ready, 0, a.err);
       tc_fence_after();
-      auto issue_s = [&](int j) {
-        const uint32_t ks = kv_s + (j % kStages) * kStageBytes;
-        const uint32_t d = tmem + (uint32_t)((j & 1) * kTileKeys);
+      // S of pair q: M = 128 rows, N = 128 keys (64 for a last single tile),
+      // K = D; the B operand is the pair's K sub-tiles.
+      auto issue_s = [&](int q) {
+        const int nt = min(2, n - 2 * q);
+        const uint32_t kb = k_chunk(2 * q, 0);
+        const uint32_t d = tmem + (uint32_t)((q & 1) * kPairKeys);
+        const uint32_t id_s = idesc_bf16(kRows, nt * kTileKeys, false);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint64_t ad = sw128_desc(q_s + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
-          const uint64_t bd = sw128_desc(ks + (kk / 4) * kKVSub + (kk % 4) * 32, 16, 1024);
+          const uint64_t bd = sw128_desc(kb + (kk / 4) * kPairSub + (kk % 4) * 32, 16, 1024);
           tc_mma(d, ad, bd, id_s, kk > 0);
         }
-        tc_commit(&s_full[j & 1]);
+        tc_commit(&s_full[q & 1]);
       };
-      auto issue_pv = [&](int j) {
-        const uint32_t ps = kPInK ? kv_s + (j % kStages) * kStageBytes : p_s + (j & 1) * kQBytes;
-        const uint32_t vs = kv_s + (j % kStages) * kStageBytes + kSub * kKVSub;
+      // O += P V over the pair's keys, 16 keys per instruction.
+      auto issue_pv = [&](int q) {
+        const int nk = 4 * min(2, n - 2 * q);
+        const uint32_t pb = p_block(q);
+        const uint32_t vb = v_chunk(2 * q, 0);
 #pragma unroll
-        for (int kk = 0; kk < kTileKeys / 16; ++kk) {
-          const uint64_t ad = sw128_desc(ps + kk * 32, 16, 1024);
-          const uint64_t bd = sw128_desc(vs + kk * 16 * 128, kKVSub, 1024);
-          tc_mma(tmem + kOCol, ad, bd, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < 8; ++kk) {
+          if (kk >= nk) break;
+          const uint64_t ad = sw128_desc(pb + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
+          const uint64_t bd = sw128_desc(vb + kk * 16 * 128, kPairSub, 1024);
+          tc_mma(tmem + kOCol, ad, bd, id_o, (q > 0 || kk > 0) ? 1u : 0u);
         }
-        tc_commit(&pv_done[j & 1]);
-        tc_commit(&kv_empty[j % kStages]);
+        tc_commit(&pv_done[q & 1]);
+        tc_commit(&kv_empty[q % kPairs]);
       };
-      // In order: S_{j+1} is issued before waiting for P_j, so the scores of
-      // the next tile are computed while the softmax of this one runs; and
-      // since S_{j+1} is issued after PV_{j-1}, the completion of S_{j+1}
-      // (s_full) implies PV_{j-1} is done, which keeps every later parity
+      // In order: S_{q+1} is issued before waiting for P_q, so the scores of
+      // the next pair are computed while the softmax of this one runs; and
+      // since S_{q+1} is issued after PV_{q-1}, the completion of S_{q+1}
+      // (s_full) implies PV_{q-1} is done, which keeps every later parity
       // wait on pv_done at most one phase behind.
-      auto wait_issue_s = [&](int j) -> bool {
-        if (!mbar_wait(&kv_full[j % kStages], (j / kStages) & 1, a.err)) return false;
-        if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1, a.err)) return false;
+      auto wait_issue_s = [&](int q) -> bool {
+        const int j0 = 2 * q, nt = min(2, n - j0);
+        for (int e = 0; e < nt; ++e)
+          if (!mbar_wait(&kv_full[(j0 + e) % kStages], ((j0 + e) / kStages) & 1, a.err)) return false;
+        if (!mbar_wait(&s_free[q & 1], ((q >> 1) & 1) ^ 1, a.err)) return false;
         tc_fence_after();
-        issue_s(j);
+        issue_s(q);
         return true;
       };
       if (ok) ok = wait_issue_s(0);
-      // (Issuing PV_j ahead of S_{j+1} when P_j is ready first measured
-      // slower: the next tile's softmax then waits longer for its scores.)
-      for (int j = 0; j < n && ok; ++j) {
-        if (j + 1 < n && !wait_issue_s(j + 1)) break;
-        if (!mbar_wait(&p_full[j & 1], (j >> 1) & 1, a.err)) break;
+      // (Issuing PV_q ahead of S_{q+1} when P_q is ready first measured
+      // slower: the next softmax then waits longer for its scores.)
+      for (int q = 0; q < np && ok; ++q) {
+        if (q + 1 < np && !wait_issue_s(q + 1)) break;
+        if (!mbar_wait(&p_full[q & 1], (q >> 1) & 1, a.err)) break;
         tc_fence_after();
-        issue_pv(j);
+        issue_pv(q);
       }
     }
   } else {
     // ------------------------------------------------ softmax warps
-    constexpr int kCW = kTileKeys / (2 * R);     // columns per warp: 32 or 16
+    constexpr int kCW = kPairKeys / (2 * R);     // columns per warp: 64 or 32
     constexpr int kRowsPerCopy = kRows / R;
     constexpr int kGroupThreads = 64 * R;        // the warps that share a row
     const int sw = warp - 2;                     // 0..7
@@ -379,12 +418,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int lane_t = quad * 32 + lane;         // TMEM lane
     const int row = lane_t % kRowsPerCopy;       // packed row
     const int dup = lane_t / kRowsPerCopy;       // copy of the row (R = 2)
-    const int cbase = kCW * (dup * 2 + sub);     // this warp's columns of a tile
+    const int cbase = kCW * (dup * 2 + sub);     // this warp's columns of a pair
+    const int half = cbase / kTileKeys;          // ... all inside one tile
+    const int coff = cbase % kTileKeys;          // first column inside that tile
     const bool owns_o = dup == 0;                // O row `row` lives in this lane
     const int bar_id = 1 + (R == 1 ? quad : (quad & 1));
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     // softmax warp index of (quadrant q, sub s)
-    auto sw_of = [](int q, int s_) { return 4 * s_ + ((q - 2) & 3); };
+    auto sw_of = [](int q_, int s_) { return 4 * s_ + ((q_ - 2) & 3); };
     // Q row -> shared (swizzled, K-major); each sub-warp copies half a row;
     // padding rows are zero.
     {
@@ -402,38 +443,46 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
-    // Every softmax warp runs all n iterations and meets its group barrier
+    // Every softmax warp runs all np iterations and meets its group barrier
     // once per iteration, also after a bounded wait gave up (then it only
     // keeps the barrier count), so that no named barrier waits forever.
-    for (int j = 0; j < n; ++j) {
+    for (int q = 0; q < np; ++q) {
+      const int j = 2 * q + half;                // the tile this warp's columns are in
       const int t = t_begin + j;
-      int valid = t < n_cache_tiles ? min(kTileKeys, len - t * kTileKeys) : a.k;
-      // causal rows of the block see the block keys j <= i only
-      if (t >= n_cache_tiles && row / a.G < a.n_causal) valid = row / a.G + 1;
-      if (ok && !mbar_wait(&s_full[j & 1], (j >> 1) & 1, a.err)) ok = false;
+      int valid;
+      if (j >= n) {
+        valid = 0;                               // a last pair of one tile
+      } else if (t < n_cache_tiles) {
+        valid = min(kTileKeys, len - t * kTileKeys);
+      } else {
+        // causal rows of the block see the block keys j <= i only
+        valid = row / a.G < a.n_causal ? row / a.G + 1 : a.k;
+      }
+      if (ok && !mbar_wait(&s_full[q & 1], (q >> 1) & 1, a.err)) ok = false;
       // tcgen05.ld/st are warp-collective: the warp goes on only as a whole
       ok = __all_sync(0xffffffffu, ok);
       float s[kCW];
       float mloc = -INFINITY;
       if (ok) {
         tc_fence_after();
-        const uint32_t sa = tmem + lane_addr + (uint32_t)((j & 1) * kTileKeys + cbase);
+        const uint32_t sa = tmem + lane_addr + (uint32_t)((q & 1) * kPairKeys + cbase);
+        uint32_t r[kCW / 16][16];
 #pragma unroll
-        for (int h = 0; h < kCW / 16; ++h) {
-          uint32_t r[16];
-          tc_ld16(sa + 16 * h, r);
-          tc_wait_ld();
+        for (int h = 0; h < kCW / 16; ++h) tc_ld16(sa + 16 * h, r[h]);
+        tc_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 16; ++e) s[16 * h + e] = __uint_as_float(r[e]);
-        }
+        for (int h = 0; h < kCW / 16; ++h)
+#pragma unroll
+          for (int e = 0; e < 16; ++e) s[16 * h + e] = __uint_as_float(r[h][e]);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&s_free[j & 1]);
-        // masked keys only exist in the last cache tile and the block tile
-        if (valid < cbase + kCW) {
+        if (lane == 0) mbar_arrive(&s_free[q & 1]);
+        // masked keys only exist in the last cache tile, the block tile and
+        // the empty half of a last single-tile pair
+        if (valid < coff + kCW) {
 #pragma unroll
           for (int c = 0; c < kCW; ++c)
-            if (cbase + c >= valid) s[c] = -INFINITY;
+            if (coff + c >= valid) s[c] = -INFINITY;
         }
         float mx[8];
 #pragma unroll
@@ -448,7 +497,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       // The group agrees on max_w(round_up_bf16(m_w)) >= the row maximum: a
       // reference at or above the maximum is all the lazy rescale needs (l and
       // O share it), and every warp of the group takes the same value.
-      red_max[((j & 1) * kSoftWarps + sw) * 32 + lane] = bf16_bits_round_up(mloc);
+      red_max[((q & 1) * kSoftWarps + sw) * 32 + lane] = bf16_bits_round_up(mloc);
       asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
       if (!ok) continue;
       float mraw = -INFINITY;
@@ -457,17 +506,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
         for (int s2 = 0; s2 < 2; ++s2) {
           const int w2 = sw_of((quad & 1) + 2 * d2 + (R == 1 ? (quad & 2) : 0), s2);
-          mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((j & 1) * kSoftWarps + w2) * 32 + lane]));
+          mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((q & 1) * kSoftWarps + w2) * 32 + lane]));
         }
       const float mt = mraw * a.scale_log2;     // the scale is positive
       // Each row decides for itself; the TMEM rescale of O is warp-collective,
       // so a warp rescales when any of its rows does (alpha = 1 for the rest).
       const bool rescale = m_ref != -INFINITY && mt > m_ref + kRescaleThreshold;
       const bool warp_rescale = __any_sync(0xffffffffu, rescale);
-      // The P buffer of this tile is free once PV(j-2) is done; O itself is
-      // only touched (rescaled) after PV(j-1).
-      const int wait_j = (warp_rescale && owns_o) ? j - 1 : (kPInK ? -1 : j - 2);
-      bool waited = wait_j < 0 || mbar_wait(&pv_done[wait_j & 1], (wait_j >> 1) & 1, a.err);
+      // The P block of this pair is free once PV(q-2) is done (it lives in
+      // the pair's own K sub-tiles for D = 128); O itself is only touched
+      // (rescaled) after PV(q-1).
+      const int wait_q = (warp_rescale && owns_o) ? q - 1 : (kPInK ? -1 : q - 2);
+      bool waited = wait_q < 0 || mbar_wait(&pv_done[wait_q & 1], (wait_q >> 1) & 1, a.err);
       if (!__all_sync(0xffffffffu, waited)) {
         ok = false;
         continue;
@@ -494,10 +544,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         tc_wait_st();
       }
       // P = 2^(scale * s - m_ref) as bf16 into this warp's columns of the
-      // tile's P buffer (row `row`).  Rows past M and, with R = 2, rows 64+
+      // pair's P block (row `row`).  Rows past M and, with R = 2, rows 64+
       // of P are never written: their O rows are garbage that is never read.
-      const uint32_t pb =
-          kPInK ? kv_s + (j % kStages) * kStageBytes : p_s + (j & 1) * kQBytes;
+      const uint32_t pb = p_block(q) + half * kQBytes;
       {
         const float nm = -m_ref;
         float psum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -509,7 +558,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
             p[e] = exp2f(fmaf(s[c * 8 + e], a.scale_log2, nm));
             psum[e] += p[e];
           }
-          st_shared_v4(swz(pb, row, cbase / 8 + c),
+          st_shared_v4(swz(pb, row, coff / 8 + c),
                        make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7])));
         }
@@ -518,12 +567,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[j & 1]);
+      if (lane == 0) mbar_arrive(&p_full[q & 1]);
     }
     grid_dependents_launch();
     // ------------------------------------------------ epilogue
     // Row sums over the group, in a fixed order.  The first barrier lets the
-    // group finish reading the last tile's maxima before the buffer is reused.
+    // group finish reading the last pair's maxima before the buffer is reused.
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
     red_l[sw * 32 + lane] = l;
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
@@ -536,7 +585,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const bool mine = owns_o && row < a.M;
     // the two sub-warps of the row's quadrant write half of the D columns each
     const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
-    bool final_ok = ok && n > 0 && owns_o && mbar_wait(&pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, a.err);
+    bool final_ok =
+        ok && np > 0 && owns_o && mbar_wait(&pv_done[(np - 1) & 1], ((np - 1) >> 1) & 1, a.err);
     final_ok = __all_sync(0xffffffffu, final_ok);   // the reads below are warp-collective
     if (final_ok) {
       tc_fence_after();
@@ -604,9 +654,9 @@ namespace sbd {
 size_t attn_tc_smem_bytes(int D) {
   const int sub = D / 64;
   const bool p_in_k = D == 128;
-  const int stages = p_in_k ? 6 : 5;
-  return 1024 + (size_t)sub * kRows * 128 + (p_in_k ? 0 : 2 * kRows * 128) +
-         (size_t)stages * 2 * sub * kTileKeys * 128;
+  const int pairs = p_in_k ? 3 : 4;
+  return 1024 + (size_t)sub * kRows * 128 + (p_in_k ? 0 : 4 * kRows * 128) +
+         (size_t)pairs * 2 * sub * kPairKeys * 128;
 }
 
 sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
@@ -647,3 +697,4 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
 }
 
 }  // namespace sbd
+
