@@ -47,9 +47,12 @@ constexpr int kMaxStages = 4;
 #define SBD_ATTN_KG_MT4 1
 #endif
 // bf16 attention on the tcgen05 kernel (block_attention_tc.cu) rather than
-// the mma.sync kernel of this file.
+// the mma.sync kernel of this file, from this many packed rows on.
 #ifndef SBD_ATTN_TC
 #define SBD_ATTN_TC 1
+#endif
+#ifndef SBD_ATTN_TC_MIN_ROWS
+#define SBD_ATTN_TC_MIN_ROWS 17
 #endif
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -703,11 +706,12 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.part_o = (float*)ws;
   a.part_lse = p.splits > 1 ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
 
-  // Up to 32 packed rows the mma.sync kernel measures faster (the tcgen05
-  // kernel pads every tile to 128 rows, and a TMEM lane quadrant -- 32 rows
-  // -- is read by the warps of one SM sub-partition only, so 32 rows leave
-  // the softmax to one sub-partition); above, tcgen05.
-  if (SBD_ATTN_TC && p.M > 32) {
+  // Up to 16 packed rows the mma.sync kernel measures faster (the tcgen05
+  // kernel pads every tile to 128 rows); from 17 on, tcgen05, with every row
+  // copied into 4, 2 or 1 TMEM lane quadrants so that all SM sub-partitions
+  // share the softmax.  Batch 16, KV 8192: 32 rows (k = 8) 115 -> 110 us;
+  // 16 rows (k = 4) 104 us on mma.sync against 108 us on tcgen05.
+  if (SBD_ATTN_TC && p.M >= SBD_ATTN_TC_MIN_ROWS) {
     s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, kc_app, vc_app,
                        st);
     if (s != SBD_OK) return s;

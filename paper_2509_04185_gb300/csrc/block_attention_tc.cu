@@ -179,9 +179,10 @@ struct TcArgs {
 // lives in TMEM lane r, and the two warps of its lane quadrant take 64 of the
 // pair's 128 columns each (one tile each).  R = 2 (M <= 64): rows are also
 // copied to lanes 64 + r (the MMA pads to 128 rows anyway), so four warps on
-// all four SM sub-partitions share a row, 32 columns each.  The warps sharing
-// a row exchange their partial maxima through shared memory at a named
-// barrier and take identical decisions.
+// all four SM sub-partitions share a row, 32 columns each.  R = 4 (M <= 32):
+// a copy in every lane quadrant, all eight warps share a row, 16 columns
+// each.  The warps sharing a row exchange their partial maxima through shared
+// memory at a named barrier and take identical decisions.
 template <int D, int R>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
@@ -409,7 +410,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
   } else {
     // ------------------------------------------------ softmax warps
-    constexpr int kCW = kPairKeys / (2 * R);     // columns per warp: 64 or 32
+    static_assert(R == 1 || R == 2 || R == 4, "row copies");
+    constexpr int kCW = kPairKeys / (2 * R);     // columns per warp: 64, 32 or 16
+    constexpr int kQuadStride = 4 / R;           // lane quadrants between copies of a row
     constexpr int kRowsPerCopy = kRows / R;
     constexpr int kGroupThreads = 64 * R;        // the warps that share a row
     const int sw = warp - 2;                     // 0..7
@@ -422,10 +425,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int half = cbase / kTileKeys;          // ... all inside one tile
     const int coff = cbase % kTileKeys;          // first column inside that tile
     const bool owns_o = dup == 0;                // O row `row` lives in this lane
-    const int bar_id = 1 + (R == 1 ? quad : (quad & 1));
+    const int bar_id = 1 + quad % kQuadStride;  // one named barrier per row group
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     // softmax warp index of (quadrant q, sub s)
     auto sw_of = [](int q_, int s_) { return 4 * s_ + ((q_ - 2) & 3); };
+    // quadrant of copy d of this lane's row
+    auto quad_of = [&](int d) { return quad % kQuadStride + kQuadStride * d; };
     // Q row -> shared (swizzled, K-major); each sub-warp copies half a row;
     // padding rows are zero.
     {
@@ -505,7 +510,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       for (int d2 = 0; d2 < R; ++d2)
 #pragma unroll
         for (int s2 = 0; s2 < 2; ++s2) {
-          const int w2 = sw_of((quad & 1) + 2 * d2 + (R == 1 ? (quad & 2) : 0), s2);
+          const int w2 = sw_of(quad_of(d2), s2);
           mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((q & 1) * kSoftWarps + w2) * 32 + lane]));
         }
       const float mt = mraw * a.scale_log2;     // the scale is positive
@@ -581,7 +586,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     for (int d2 = 0; d2 < R; ++d2)
 #pragma unroll
       for (int s2 = 0; s2 < 2; ++s2)
-        lsum += red_l[sw_of((quad & 1) + 2 * d2 + (R == 1 ? (quad & 2) : 0), s2) * 32 + lane];
+        lsum += red_l[sw_of(quad_of(d2), s2) * 32 + lane];
     const bool mine = owns_o && row < a.M;
     // the two sub-warps of the row's quadrant write half of the D columns each
     const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
@@ -685,9 +690,15 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t smem = attn_tc_smem_bytes(p.D);
-  const bool rep2 = p.M <= kRows / 2;
-  const void* fn = p.D == 128 ? (rep2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>)
-                              : (rep2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>);
+  // copies of every packed row in the 128 MMA rows: 4, 2 or 1
+  const int R = p.M <= kRows / 4 ? 4 : (p.M <= kRows / 2 ? 2 : 1);
+  const void* fn;
+  if (p.D == 128)
+    fn = R == 4 ? (const void*)attn_tc_kernel<128, 4>
+                : (R == 2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>);
+  else
+    fn = R == 4 ? (const void*)attn_tc_kernel<64, 4>
+                : (R == 2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>);
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
   CUtensorMap k_map = tk, v_map = tv;

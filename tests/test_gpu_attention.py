@@ -61,8 +61,8 @@ BF16 = gen.get_workload("llama8b_k16")
 
 
 @pytest.mark.parametrize("D", [64, 128])
-@pytest.mark.parametrize("G,k", [(4, 1), (4, 4), (4, 8), (1, 16), (4, 12), (4, 16), (2, 40 // 2),
-                                 (4, 32), (8, 16)])
+@pytest.mark.parametrize("G,k", [(4, 1), (4, 4), (1, 16), (4, 8), (3, 7), (2, 9), (4, 12), (4, 16),
+                                 (2, 40 // 2), (4, 32), (8, 16)])
 def test_bf16_shapes(sbd, D, G, k):
     Hkv = 2
     w = gen.shrink(BF16, batch=2, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv, head_dim=D,
