@@ -38,6 +38,10 @@ constexpr int kMaxStages = 16;
 // A pipeline stage holds up to this many consecutive boxes along the hidden
 // dimension (longer contiguous reads of every W row per stage), and the ring
 // gets this many bytes of shared memory.
+// Hidden rows are loaded in boxes of up to 128 rows (1), or of 16 only (0).
+#ifndef SBD_HEAD_BIG_BOXES
+#define SBD_HEAD_BIG_BOXES 1
+#endif
 #ifndef SBD_HEAD_MAX_BOXES
 #define SBD_HEAD_MAX_BOXES 4
 #endif
@@ -324,6 +328,7 @@ struct HeadArgs {
   int n_acc;            // accumulator buffers in tensor memory (2, or 1 above 256 rows)
   uint32_t tmem_cols;
   float tau;
+  int h_big;            // tallest hidden-row box encoded: 16, 64 or 128 rows
 };
 
 // kPhilox: the Gumbel noise is generated in the epilogue (philox.cuh)
@@ -331,7 +336,9 @@ struct HeadArgs {
 template <bool kPhilox>
 __global__ void __launch_bounds__(kHeadThreads, SBD_HEAD_CTAS_PER_SM)
 head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
-               const __grid_constant__ CUtensorMap tmap_h, const HeadArgs a) {
+               const __grid_constant__ CUtensorMap tmap_h,
+               const __grid_constant__ CUtensorMap tmap_h64,
+               const __grid_constant__ CUtensorMap tmap_h128, const HeadArgs a) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
@@ -427,10 +434,18 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
               (void)policy;
               tma_load_2d(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM);
 #endif
-              // hidden rows in boxes of 16: only the n_eff rows the MMA reads
-              for (int r0 = 0; r0 < n_eff; r0 += 16)
-                tma_load_2d(st + boxes * kABytes + x * b_box + r0 * 128, &tmap_h, &full_bar[s],
-                            col, r0);
+              // the n_eff hidden rows the MMA reads, in the tallest boxes that
+              // fit: these rows come from L2 for every vocabulary tile, where
+              // the copy rate per SM grows with the box size
+              uint8_t* hb = st + boxes * kABytes + x * b_box;
+              int r0 = 0;
+              if (a.h_big >= 128)
+                for (; r0 + 128 <= n_eff; r0 += 128)
+                  tma_load_2d(hb + r0 * 128, &tmap_h128, &full_bar[s], col, r0);
+              if (a.h_big >= 64)
+                for (; r0 + 64 <= n_eff; r0 += 64)
+                  tma_load_2d(hb + r0 * 128, &tmap_h64, &full_bar[s], col, r0);
+              for (; r0 < n_eff; r0 += 16) tma_load_2d(hb + r0 * 128, &tmap_h, &full_bar[s], col, r0);
             }
           }
         }
@@ -796,7 +811,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
   cudaError_t e;
   int* err = device_error_word();
   if (p.bf16) {
-    CUtensorMap tw, th;
+    CUtensorMap tw, th, th64, th128;
     {
       const uint64_t dims[2] = {(uint64_t)p.H, (uint64_t)p.V};
       const uint64_t strides[1] = {(uint64_t)p.H * 2};
@@ -812,6 +827,20 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
       s = encode_tensor_map(&th, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)W.hidden_c, dims,
                             strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
       if (s != SBD_OK) return s;
+      th64 = th;
+      th128 = th;
+      if (p.rows_alloc >= 64) {
+        const uint32_t box64[2] = {(uint32_t)kBK, 64u};
+        s = encode_tensor_map(&th64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)W.hidden_c, dims,
+                              strides, box64, CU_TENSOR_MAP_SWIZZLE_128B);
+        if (s != SBD_OK) return s;
+      }
+      if (p.rows_alloc >= 128) {
+        const uint32_t box128[2] = {(uint32_t)kBK, 128u};
+        s = encode_tensor_map(&th128, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)W.hidden_c,
+                              dims, strides, box128, CU_TENSOR_MAP_SWIZZLE_128B);
+        if (s != SBD_OK) return s;
+      }
     }
     HeadArgs a;
     a.gumbel = gumbel;
@@ -828,6 +857,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.H = p.H;
     a.rows_alloc = p.rows_alloc;
     a.n_tiles = (p.V + kBM - 1) / kBM;
+    a.h_big = SBD_HEAD_BIG_BOXES ? (p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16)) : 16;
     a.ring_bytes = head_ring_bytes(p.rows_alloc);
     a.n_acc = 2 * p.rows_alloc <= 512 ? 2 : 1;
     uint32_t cols = 32;
@@ -838,7 +868,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     const void* fn = philox ? (const void*)head_tc_kernel<true> : (const void*)head_tc_kernel<false>;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
-    void* args[] = {(void*)&tw, (void*)&th, (void*)&a};
+    void* args[] = {(void*)&tw, (void*)&th, (void*)&th64, (void*)&th128, (void*)&a};
     s = launch_pdl(fn, dim3(p.n_ctas), dim3(kHeadThreads), smem, st, args,
                    "head_tc_kernel launch");
     if (s != SBD_OK) return s;
