@@ -74,6 +74,22 @@ def test_bf16_shapes(sbd, B, k, V, H, tau):
     assert compare_head(d, "bf16", tau, ent, tok, with_noise=tau != 0.0) <= 1
 
 
+@pytest.mark.parametrize("R", [64, 80, 128, 144, 192, 208, 256, 320])
+def test_bf16_hidden_box_decomposition(sbd, R):
+    """Exactly R masked rows out of 512: the live rows are loaded in boxes of
+    128, 64 and 16 rows (144 = 128 + 16, 208 = 128 + 64 + 16; above 256 the
+    MMA N splits); every row must come out right."""
+    w = gen.shrink(gen.get_workload("llama8b_k16"), batch=16, block_k=32, vocab=1100, hidden=192,
+                   cache_len=16)
+    d = step_inputs(w, seed=R)
+    rng = np.random.default_rng(R)
+    m = np.zeros(16 * 32, dtype=np.uint8)
+    m[rng.choice(16 * 32, size=R, replace=False)] = 1
+    d["masked"] = m.reshape(16, 32)
+    ent, tok = run_head(sbd, d, "bf16", 1.0)
+    assert compare_head(d, "bf16", 1.0, ent, tok) <= max(1, R // 50)
+
+
 def test_bf16_all_masked_and_none_masked(sbd):
     w = gen.shrink(gen.get_workload("llama8b_k16"), batch=4, block_k=8, vocab=1500, hidden=256)
     d = step_inputs(w, seed=5)
