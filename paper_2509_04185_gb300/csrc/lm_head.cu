@@ -75,6 +75,13 @@ constexpr int kHeadThreads = 64 + kEpiThreads;   // warp 0 TMA, warp 1 MMA, then
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
+// Shared-memory scratch of the tensor-core epilogue for `rows` hidden rows:
+// per TMEM quadrant and row the running (m, S, T, best) and best id, then
+// the row map; rounded to 1 KB.
+__host__ __device__ constexpr int head_scratch_bytes(int rows) {
+  return (4 * rows * (16 + 4) + rows * 4 + 1023) & ~1023;
+}
+
 // ------------------------------------------------------------ tcgen05 PTX
 __device__ __forceinline__ void tc_alloc(uint32_t* dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -349,18 +356,6 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (sbase - smem_u32(smem_raw));
-  // epilogue scratch first, then the ring
-  uint8_t* ep = gbase;
-  const int ep_bytes = (4 * a.rows_alloc * (16 + 4) + a.rows_alloc * 4 + 1023) & ~1023;
-  uint8_t* ring = gbase + ep_bytes;
-  const uint32_t rbase = sbase + ep_bytes;
-  StatsRef wstats[4];
-  for (int w = 0; w < 4; ++w) {
-    wstats[w].msTb = reinterpret_cast<float4*>(ep) + w * a.rows_alloc;
-    wstats[w].idx = reinterpret_cast<int*>(ep + (size_t)4 * a.rows_alloc * sizeof(float4)) +
-                    w * a.rows_alloc;
-  }
-  int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * a.rows_alloc * (sizeof(float4) + 4));
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmap_w);
@@ -371,15 +366,32 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   grid_dependency_wait();
   const int R = *a.n_rows;
   const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
+  // Epilogue scratch for the n_eff live rows first, then the ring, which
+  // also gets what the allocation kept for the scratch of rows_alloc rows.
+  uint8_t* ep = gbase;
+  const int ep_bytes = head_scratch_bytes(n_eff);
+  const int ring_bytes = a.ring_bytes + head_scratch_bytes(a.rows_alloc) - ep_bytes;
+  uint8_t* ring = gbase + ep_bytes;
+  const uint32_t rbase = sbase + ep_bytes;
+  StatsRef wstats[4];
+  for (int w = 0; w < 4; ++w) {
+    wstats[w].msTb = reinterpret_cast<float4*>(ep) + w * n_eff;
+    wstats[w].idx = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * sizeof(float4)) + w * n_eff;
+  }
+  int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * (sizeof(float4) + 4));
   // Ring shape from the actual row count: a stage holds `boxes` 64-column
-  // boxes of W (16 KB each) and of the n_eff hidden rows; as many boxes as
-  // still leave 3 stages, then as many stages as fit.
+  // boxes of W (16 KB each) and of the n_eff hidden rows.  Above two boxes,
+  // as many as still leave 3 stages; two boxes as long as 2 stages fit;
+  // then as many stages as fit.  (Two boxes in 2 stages measured faster
+  // than one box in 4-5: 160 rows 233 -> 219 us, 256 rows 255 -> 249 us;
+  // four boxes in 2 stages slower than two in 4 at 60 rows.)
   const int b_box = n_eff * kBK * 2;
+  auto fits = [&](int bx, int n_st) { return ring_bytes / (bx * (kABytes + b_box)) >= n_st; };
   int boxes = SBD_HEAD_MAX_BOXES;
-  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || a.ring_bytes / (boxes * (kABytes + b_box)) < 3))
+  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || !fits(boxes, boxes > 2 ? 3 : 2)))
     boxes >>= 1;
   const int stage_bytes = boxes * (kABytes + b_box);     // [A boxes | B boxes]
-  int stages = a.ring_bytes / stage_bytes;
+  int stages = ring_bytes / stage_bytes;
   if (stages > kMaxStages) stages = kMaxStages;
   // Epilogue warps with a chunk of 16 columns to reduce, per TMEM quadrant;
   // the others skip the tile loop.
@@ -398,7 +410,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   }
   if (warp >= 2) {
     const int te = threadIdx.x - 64;
-    for (int i = te; i < a.rows_alloc; i += kEpiThreads) {
+    for (int i = te; i < n_eff; i += kEpiThreads) {
       rmap[i] = i < R ? a.row_map[i] : 0;
       for (int w = 0; w < 4; ++w) store_stats(wstats[w], i, rowstats_empty());
     }
@@ -744,21 +756,18 @@ HeadWs head_ws_layout(const sbd::HeadPlan& p, void* base) {
   return w;
 }
 
-int head_ep_bytes(int rows_alloc) {
-  return (4 * rows_alloc * (16 + 4) + rows_alloc * 4 + 1023) & ~1023;
-}
 
 // Shared memory of the ring: SBD_HEAD_RING_BYTES per SM, within what a CTA
 // can have next to the epilogue scratch.
 int head_ring_bytes(int rows_alloc) {
   const int per_cta = (224 * 1024) / SBD_HEAD_CTAS_PER_SM - 1024 - 1024;
   int budget = SBD_HEAD_RING_BYTES / SBD_HEAD_CTAS_PER_SM;
-  if (budget > per_cta - head_ep_bytes(rows_alloc)) budget = per_cta - head_ep_bytes(rows_alloc);
+  if (budget > per_cta - head_scratch_bytes(rows_alloc)) budget = per_cta - head_scratch_bytes(rows_alloc);
   return budget;
 }
 
 size_t head_smem_bytes(int rows_alloc) {
-  return 1024 + (size_t)head_ep_bytes(rows_alloc) + head_ring_bytes(rows_alloc);
+  return 1024 + (size_t)head_scratch_bytes(rows_alloc) + head_ring_bytes(rows_alloc);
 }
 
 }  // namespace
