@@ -45,6 +45,25 @@ def dist_env():
             int(os.environ.get("WORLD_SIZE", "1")))
 
 
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The largest x over all ranks (a barrier follows); x itself at N = 1.
+    The timed region of every replica is reduced this way."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.barrier()
+    return float(t.item())
+
+
+def job_us_per_step(job_ms: float, steps_per_rank: int, world: int) -> float:
+    """Whole-job time per step: each of `world` replicas ran `steps_per_rank`
+    steps within `job_ms`, the slowest rank's time."""
+    return job_ms * 1000.0 / (steps_per_rank * world)
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -294,12 +313,7 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     if sampler:
         sampler.mark("timed_end")
-    total_ms = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.barrier()
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(start.elapsed_time(end), world, dev)
     n_accepted = int(n_un.sum().item())
     if sbd.sbd_device_error() != 0:
         raise RuntimeError("device error word set during the timed region")
@@ -357,8 +371,8 @@ def run_ours(args):
             e2e_step()
         e2.record(stream)
         torch.cuda.synchronize(dev)
-        e2e_ms = s2.elapsed_time(e2) / n_e2e
-        e2e = {"value": round(e2e_ms * 1000.0 / world, 3), "unit": UNIT,
+        e2e_ms = max_over_ranks(s2.elapsed_time(e2), world, dev) / n_e2e
+        e2e = {"value": round(job_us_per_step(e2e_ms, 1, world), 3), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "steps": n_e2e}
 
@@ -375,7 +389,7 @@ def run_ours(args):
     attn_gbs = ab["attention"] / (attn_ms * 1e-3) / 1e9
     step_bytes = ab["attention"] + ab["head"] + ab["eb"]
     ms_per_step = total_ms / args.steps
-    value_us = ms_per_step * 1000.0 / world
+    value_us = job_us_per_step(total_ms, args.steps, world)
     cpu = None
     if world == 1 and not args.skip_cpu:
         cpu = cpu_baseline(w, d, args)
@@ -658,12 +672,7 @@ def run_sweep(args):
     wall = time.perf_counter() - t0
     if sampler:
         sampler.mark("timed_end")
-    total_ms = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.barrier()
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(start.elapsed_time(end), world, dev)
     attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
@@ -680,7 +689,7 @@ def run_sweep(args):
     ms_per_step = total_ms / n_steps
     attn_gbs = attn_bytes / (attn_ms * 1e-3) / 1e9
     line = {
-        "metric": METRIC, "value": round(ms_per_step * 1000.0 / world, 3), "unit": UNIT,
+        "metric": METRIC, "value": round(job_us_per_step(total_ms, n_steps, world), 3), "unit": UNIT,
         "n_gpus": world, "steps": n_steps, "warmup": args.warmup,
         "ms_per_step": round(ms_per_step, 6), "higher_is_better": False, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
