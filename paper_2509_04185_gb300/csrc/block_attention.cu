@@ -51,6 +51,11 @@ constexpr int kMaxStages = 4;
 #ifndef SBD_ATTN_TC
 #define SBD_ATTN_TC 1
 #endif
+// Largest batch for which the CTAs of a multi-wave launch take the
+// sequences longest first (0: never).
+#ifndef SBD_ATTN_ORDER_MAX_B
+#define SBD_ATTN_ORDER_MAX_B 128
+#endif
 #ifndef SBD_ATTN_TC_MIN_ROWS
 #define SBD_ATTN_TC_MIN_ROWS 17
 #endif
@@ -101,6 +106,7 @@ struct AttnArgs {
   __nv_bfloat16* kc_app;     // writable caches for the causal rows' keys/values, or NULL
   __nv_bfloat16* vc_app;
   int B, k, Hq, Hkv, G, M, Lmax, splits, MT, KG, stages, n_causal;
+  int order;                 // blockIdx.z -> sequence by descending length
   float scale_log2;
 };
 
@@ -127,7 +133,8 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
 
   const int NW = a.MT * a.KG;                        // compute warps
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+  const int split = blockIdx.x, hkv = blockIdx.y;
+  __shared__ int b_pick;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -138,6 +145,11 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
   }
   // Everything below may read what the previous kernel on the stream wrote.
   grid_dependency_wait();
+  if (a.order) {
+    longest_first_pick(a.lens, a.B, a.Lmax, blockIdx.z, &b_pick);
+    __syncthreads();
+  }
+  const int b = a.order ? b_pick : (int)blockIdx.z;
 
   int len = a.lens[b];
   if (len < 0 || len > a.Lmax) {
@@ -621,6 +633,10 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
   } else {
     p.splits = choose_splits(p.B * p.Hkv, tiles, num_sms());
   }
+  // With more CTAs than one wave, the CTAs take the sequences longest first
+  // (the pick costs B^2 comparisons per CTA, hence the batch limit).
+  p.order = p.bf16 && p.B > 1 && p.B <= SBD_ATTN_ORDER_MAX_B &&
+            (long long)p.B * p.Hkv * p.splits > num_sms();
   // Ring depth: as many stages as a split has tiles, between 2 and 4.
   const int per_split = (tiles + p.splits - 1) / p.splits;
   const int cap = SBD_ATTN_STAGE_CAP < kMaxStages ? SBD_ATTN_STAGE_CAP : kMaxStages;
@@ -699,6 +715,7 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.KG = p.KG;
   a.stages = p.stages;
   a.n_causal = p.n_causal;
+  a.order = p.order ? 1 : 0;
   a.kc_app = (__nv_bfloat16*)kc_app;
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;

@@ -172,6 +172,7 @@ struct TcArgs {
   __nv_bfloat16* kc_app;     // writable caches for the causal rows' keys/values, or NULL
   __nv_bfloat16* vc_app;
   int B, k, Hq, Hkv, G, M, Lmax, splits, n_causal;
+  int order;                 // blockIdx.z -> sequence by descending length
   float scale_log2;
 };
 
@@ -233,7 +234,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+  const int split = blockIdx.x, hkv = blockIdx.y;
+  __shared__ int b_pick;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(&kv_full[s], 1);
@@ -251,6 +253,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // All 512 tensor-memory columns are taken only after the previous grid is
   // done, so that no CTA of it can be left waiting for them.
   grid_dependency_wait();
+  if (a.order) {
+    longest_first_pick(a.lens, a.B, a.Lmax, blockIdx.z, &b_pick);
+    __syncthreads();
+  }
+  const int b = a.order ? b_pick : (int)blockIdx.z;
   if (warp == 1) tc_alloc(&tmem_base_sh, kTmemCols);
 
   int len = a.lens[b];
@@ -686,6 +693,7 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.Lmax = p.Lmax;
   a.splits = p.splits;
   a.n_causal = p.n_causal;
+  a.order = p.order ? 1 : 0;
   a.kc_app = (__nv_bfloat16*)kc_app;
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;

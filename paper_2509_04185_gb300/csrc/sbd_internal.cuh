@@ -28,6 +28,7 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
 // validated by the API layer.
 struct AttnPlan {
   int B, k, Hq, Hkv, G, D, Lmax, M, splits, stages, MT, KG;
+  bool order;         // CTAs take sequences longest first (more than one wave)
   int n_causal;       // block rows i < n_causal see block keys j <= i only
   float scale_log2;   // softmax scale * log2(e)
   bool bf16;
@@ -137,6 +138,25 @@ __device__ __forceinline__ bool mbar_poll_parity(uint64_t* bar, uint32_t parity)
       : "memory");
   return ok != 0;
 }
+// The sequence of CTA z when a launch spans more than one wave of CTAs: the
+// one of rank z in descending cache length (ties by index), so that the
+// longest sequences start first (longest-processing-time-first list
+// scheduling of the CTAs onto the SMs).  Every thread of the CTA takes part;
+// *out_b is set by one of them, and the caller's barrier publishes it.
+// Lengths are clamped to [0, Lmax] as in the kernels.
+__device__ __forceinline__ void longest_first_pick(const int32_t* lens, int B, int Lmax, int z,
+                                                   int* out_b) {
+  for (int i = threadIdx.x; i < B; i += blockDim.x) {
+    const int li = min(max(lens[i], 0), Lmax);
+    int rank = 0;
+    for (int j = 0; j < B; ++j) {
+      const int lj = min(max(lens[j], 0), Lmax);
+      rank += (lj > li || (lj == li && j < i)) ? 1 : 0;
+    }
+    if (rank == z) *out_b = i;
+  }
+}
+
 // Waits until the phase with the given parity has completed, for at most
 // kWaitLimitNs.  Returns false (and records SBD_DEVERR_TIMEOUT) on time-out.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {

@@ -161,3 +161,16 @@ def test_growing_scores_take_the_rescale_path(sbd, G, k, splits):
     assert np.isfinite(got).all()
     assert float(np.abs(got - ref).max()) <= BF16_ATTN_TOL
     assert sbd.sbd_device_error() == 0
+
+
+@pytest.mark.parametrize("k,G", [(8, 4), (4, 4), (16, 4)])
+def test_multi_wave_launch_takes_sequences_longest_first(sbd, k, G):
+    """40 sequences x 8 KV heads = 320 CTAs, more than one wave: the CTAs
+    take the sequences in descending length, ties by index (lengths with
+    repeats and zeros here); every output must still land in its own row."""
+    rng = np.random.default_rng(k)
+    lens = rng.choice([0, 1, 63, 64, 65, 200, 333, 500], size=40).astype(np.int32)
+    lens[[3, 17, 29]] = 333                                  # ties
+    w = gen.shrink(BF16, batch=40, block_k=k, n_q_heads=8 * G, n_kv_heads=8,
+                   cache_len=(0, 512))
+    _run_and_compare(sbd, w, seed=k, lens=lens.tolist())
