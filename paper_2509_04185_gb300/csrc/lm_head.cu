@@ -332,7 +332,6 @@ struct HeadArgs {
   int* err;
   int V, H, rows_alloc, n_tiles;
   int ring_bytes;       // shared memory of the TMA ring (shaped in the kernel)
-  int n_acc;            // accumulator buffers in tensor memory (2, or 1 above 256 rows)
   uint32_t tmem_cols;
   float tau;
   int h_big;            // tallest hidden-row box encoded: 16, 64 or 128 rows
@@ -366,6 +365,11 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   grid_dependency_wait();
   const int R = *a.n_rows;
   const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
+  // Two accumulator buffers whenever two of the live width fit in the
+  // tensor memory of the launch (half of it each), so that the epilogue of
+  // one tile overlaps the MMAs of the next; one above 256 live rows.
+  const int n_acc = 2 * n_eff <= (int)a.tmem_cols ? 2 : 1;
+  const uint32_t acc_stride = a.tmem_cols / 2;
   // Epilogue scratch for the n_eff live rows first, then the ring, which
   // also gets what the allocation kept for the scratch of rows_alloc rows.
   uint8_t* ep = gbase;
@@ -475,11 +479,11 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         int it = 0, local = 0;
         bool ok = true;
         for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x, ++local) {
-          const int acc = a.n_acc == 2 ? (local & 1) : 0;
-          const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
+          const int acc = n_acc == 2 ? (local & 1) : 0;
+          const uint32_t use = (uint32_t)(n_acc == 2 ? (local >> 1) : local);
           if (!mbar_wait(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + (uint32_t)(acc * a.rows_alloc);
+          const uint32_t d_tmem = tmem_base + (uint32_t)acc * acc_stride;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
             const int s = it % stages;
             const uint32_t ph = (it / stages) & 1;
@@ -514,12 +518,12 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
       for (int tile = blockIdx.x; sub < n_sub && tile < a.n_tiles; tile += gridDim.x, ++local) {
-        const int acc = a.n_acc == 2 ? (local & 1) : 0;
-        const uint32_t use = (uint32_t)(a.n_acc == 2 ? (local >> 1) : local);
+        const int acc = n_acc == 2 ? (local & 1) : 0;
+        const uint32_t use = (uint32_t)(n_acc == 2 ? (local >> 1) : local);
         const int v0 = tile * kBM + quad * 32;
         const int v = v0 + lane;
         const bool valid = v < a.V;
-        const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)(acc * a.rows_alloc);
+        const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)acc * acc_stride;
         // Gumbel noise of the first kGAhead chunks is loaded while the MMAs
         // run; each chunk's reduction then loads the chunk kGAhead further on.
         const int stride = 16 * n_sub;
@@ -868,9 +872,11 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.n_tiles = (p.V + kBM - 1) / kBM;
     a.h_big = SBD_HEAD_BIG_BOXES ? (p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16)) : 16;
     a.ring_bytes = head_ring_bytes(p.rows_alloc);
-    a.n_acc = 2 * p.rows_alloc <= 512 ? 2 : 1;
+    // tensor memory for two accumulators of the allocated width (one of it
+    // above 256 rows); the kernel picks the buffer count from the live rows
+    const int n_acc_alloc = 2 * p.rows_alloc <= 512 ? 2 : 1;
     uint32_t cols = 32;
-    while (cols < (uint32_t)(a.n_acc * p.rows_alloc)) cols <<= 1;
+    while (cols < (uint32_t)(n_acc_alloc * p.rows_alloc)) cols <<= 1;
     a.tmem_cols = cols;
     a.tau = tau;
     const size_t smem = head_smem_bytes(p.rows_alloc);
