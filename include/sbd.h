@@ -194,6 +194,31 @@ sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t voc
                              uint64_t seed, uint64_t offset, float* out, void* stream);
 
 /* ------------------------------------------------------------------------
+ * A plain linear layer on the LM-head kernel: y = x W^T, the GEMMs of a
+ * transformer layer at decode shapes (few rows, weights streamed once).
+ * Used to time full forwards of a model around the block step (the
+ * paper's timing section models the linear layers as GEMMs); it is not
+ * part of the block step itself.
+ *
+ *   x [rows, in_features]           bf16, row-major (device)
+ *   w [out_features, in_features]   bf16, row-major, nn.Linear layout (device)
+ *   y [rows, out_features]          bf16, row-major (device, written)
+ *
+ * y is the fp32 sum over in_features of the bf16 products, rounded to
+ * bf16 (round to nearest even).  All pointers 16-byte aligned, caller-owned;
+ * no workspace.  Asynchronous on `stream`.
+ * Supported: dtype bf16, 0 <= rows <= 512, in_features a positive multiple
+ * of 64, out_features >= 1; SBD_ERR_UNSUPPORTED otherwise.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int32_t rows, in_features, out_features;
+  sbd_dtype dtype;
+} sbd_linear_desc;
+
+sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
+                      void* stream);
+
+/* ------------------------------------------------------------------------
  * No-allocation variant of sbd_head_entropy_sample.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory -- a host framework that owns the whole device memory pool,

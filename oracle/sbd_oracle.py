@@ -480,6 +480,13 @@ def roofline_linear(block: int, batch: int, c=ROOFLINE_H100) -> float:
     return sum(roofline_gemm(m, n, k, c)[0] for (m, n, k) in shapes)
 
 
+def linear(x, w):
+    """y = x W^T in fp64 over the given values (x [T, K], W [N, K], the
+    nn.Linear layout): the GEMM of a linear layer, which the timing section
+    counts in every forward besides the attention."""
+    return np.asarray(x, np.float64) @ np.asarray(w, np.float64).T
+
+
 def roofline_forward(block: int, kv_len: int, batch: int, c=ROOFLINE_H100) -> float:
     """Forward time of one layer for a block of `block` tokens per sequence:
     attention plus the linear layers (the layer count cancels in ratios)."""

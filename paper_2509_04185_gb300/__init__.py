@@ -49,6 +49,7 @@ EXPORTS = (
     "sbd_head_entropy_confidence_sample",
     "sbd_head_entropy_sample_philox",
     "sbd_gumbel_philox",
+    "sbd_linear",
     "sbd_eb_select",
     "sbd_select",
     "sbd_status_string",
@@ -70,6 +71,11 @@ class HeadDesc(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("block_k", ctypes.c_int32),
                 ("hidden", ctypes.c_int32), ("vocab", ctypes.c_int32),
                 ("dtype", ctypes.c_int32)]
+
+
+class LinearDesc(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int32), ("in_features", ctypes.c_int32),
+                ("out_features", ctypes.c_int32), ("dtype", ctypes.c_int32)]
 
 
 class SbdError(RuntimeError):
@@ -108,6 +114,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_head_entropy_sample_philox.restype = ctypes.c_int
     lib.sbd_gumbel_philox.argtypes = [i32, vp, i32, u64, u64, vp, vp]
     lib.sbd_gumbel_philox.restype = ctypes.c_int
+    lib.sbd_linear.argtypes = [ctypes.POINTER(LinearDesc), vp, vp, vp, vp]
+    lib.sbd_linear.restype = ctypes.c_int
     lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
     lib.sbd_eb_select.restype = ctypes.c_int
     lib.sbd_select.argtypes = [i32, i32, i32, vp, vp, vp, f32, vp, vp, vp, vp]
@@ -328,6 +336,29 @@ def sbd_gumbel_philox(row_ids, vocab: int, seed: int, offset: int, out=None, *, 
     _check(lib.sbd_gumbel_philox(n, _ptr(row_ids), int(vocab), int(seed), int(offset), _ptr(out),
                                  _stream(stream)))
     return out
+
+
+def sbd_linear(x, w, out=None, *, stream=None):
+    """y = x W^T on the LM-head kernel: x [T, K] bf16, w [N, K] bf16
+    (nn.Linear layout), T <= 512, K a multiple of 64.  Returns out [T, N]
+    bf16."""
+    torch = _torch()
+    _need_cuda(x=x, w=w, out=out)
+    if x.dim() != 2 or w.dim() != 2 or x.shape[1] != w.shape[1]:
+        raise ValueError(f"shapes x {tuple(x.shape)} and w {tuple(w.shape)} do not match")
+    if out is None:
+        out = torch.empty((x.shape[0], w.shape[0]), dtype=x.dtype, device=x.device)
+    d = LinearDesc(x.shape[0], x.shape[1], w.shape[0], _dtype_code(x))
+    _check(lib.sbd_linear(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _stream(stream)))
+    return out
+
+
+def prepare_linear(x, w, out, *, stream=None) -> "Prepared":
+    """sbd_linear bound to fixed tensors (see Prepared)."""
+    _need_cuda(x=x, w=w, out=out)
+    d = LinearDesc(x.shape[0], x.shape[1], w.shape[0], _dtype_code(x))
+    args = (ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _stream(stream))
+    return Prepared(lib.sbd_linear, args, keep=(d, x, w, out))
 
 
 def sbd_head_entropy_sample_noalloc(hidden, w, masked, gumbel, tau: float, entropy, token, *,

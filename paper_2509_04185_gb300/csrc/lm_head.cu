@@ -335,11 +335,15 @@ struct HeadArgs {
   uint32_t tmem_cols;
   float tau;
   int h_big;            // tallest hidden-row box encoded: 16, 64 or 128 rows
+  __nv_bfloat16* y;     // kLinear: output [linear_rows, V]
+  int linear_rows;      // kLinear: rows of x, all live
 };
 
 // kPhilox: the Gumbel noise is generated in the epilogue (philox.cuh)
-// instead of read from a [B*k, V] buffer.
-template <bool kPhilox>
+// instead of read from a [B*k, V] buffer.  kLinear: the plain product
+// y = x W^T in bf16 (all rows of x live, no compaction, no noise); the
+// epilogue stores the accumulators instead of reducing them.
+template <bool kPhilox, bool kLinear>
 __global__ void __launch_bounds__(kHeadThreads, SBD_HEAD_CTAS_PER_SM)
 head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                const __grid_constant__ CUtensorMap tmap_h,
@@ -363,7 +367,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   if (warp == 1) tc_alloc(&tmem_base_sh, a.tmem_cols);
   // Everything below reads what the compaction kernel wrote.
   grid_dependency_wait();
-  const int R = *a.n_rows;
+  const int R = kLinear ? a.linear_rows : *a.n_rows;
   const int n_eff = R <= 16 ? 16 : ((R + 15) / 16) * 16;   // MMA N
   // Two accumulator buffers whenever two of the live width fit in the
   // tensor memory of the launch (half of it each), so that the epilogue of
@@ -415,7 +419,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   if (warp >= 2) {
     const int te = threadIdx.x - 64;
     for (int i = te; i < n_eff; i += kEpiThreads) {
-      rmap[i] = i < R ? a.row_map[i] : 0;
+      rmap[i] = (!kLinear && i < R) ? a.row_map[i] : 0;
       for (int w = 0; w < 4; ++w) store_stats(wstats[w], i, rowstats_empty());
     }
   }
@@ -514,7 +518,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       // ------------------------------------------------ epilogue warps
       const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
       const int sub = (warp - 2) / 4;          // chunks sub, sub + n_sub, ... of 16 columns
-      const bool noisy = a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
+      const bool noisy = !kLinear && a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
       for (int tile = blockIdx.x; sub < n_sub && tile < a.n_tiles; tile += gridDim.x, ++local) {
@@ -588,13 +592,23 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
           uint32_t r[16];
           tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
           tc_wait_ld();
-          float z[16];
+          if constexpr (kLinear) {
+            // y[c0 + j, v]: for each j the warp's lanes store 32 consecutive v
+            if (valid) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
-          const RowStats st = chunk16_stats(z, g, valid, a.tau, v0, lane);
-          const int col = c0 + ((lane >> 1) & 15);
-          if ((lane & 1) == 0 && col < R)
-            store_stats(wstats[quad], col, rowstats_merge(load_stats(wstats[quad], col), st));
+              for (int j = 0; j < 16; ++j)
+                if (c0 + j < R)
+                  a.y[(size_t)(c0 + j) * a.V + v] = __float2bfloat16_rn(__uint_as_float(r[j]));
+            }
+          } else {
+            float z[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
+            const RowStats st = chunk16_stats(z, g, valid, a.tau, v0, lane);
+            const int col = c0 + ((lane >> 1) & 15);
+            if ((lane & 1) == 0 && col < R)
+              store_stats(wstats[quad], col, rowstats_merge(load_stats(wstats[quad], col), st));
+          }
         }
         tc_fence_before();
         __syncwarp();
@@ -602,12 +616,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       }
       asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
       const int te = threadIdx.x - 64;
-      for (int col = te; col < R; col += kEpiThreads) {
-        RowStats s = load_stats(wstats[0], col);
-        for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats[w], col));
-        const size_t o = (size_t)blockIdx.x * a.rows_alloc + col;
-        a.part_msTb[o] = make_float4(s.m, s.S, s.T, s.best);
-        a.part_idx[o] = s.idx;
+      if constexpr (!kLinear) {
+        for (int col = te; col < R; col += kEpiThreads) {
+          RowStats s = load_stats(wstats[0], col);
+          for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats[w], col));
+          const size_t o = (size_t)blockIdx.x * a.rows_alloc + col;
+          a.part_msTb[o] = make_float4(s.m, s.S, s.T, s.best);
+          a.part_idx[o] = s.idx;
+        }
       }
     }
   }
@@ -870,6 +886,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.H = p.H;
     a.rows_alloc = p.rows_alloc;
     a.n_tiles = (p.V + kBM - 1) / kBM;
+    a.y = nullptr;
+    a.linear_rows = 0;
     a.h_big = SBD_HEAD_BIG_BOXES ? (p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16)) : 16;
     a.ring_bytes = head_ring_bytes(p.rows_alloc);
     // tensor memory for two accumulators of the allocated width (one of it
@@ -880,7 +898,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.tmem_cols = cols;
     a.tau = tau;
     const size_t smem = head_smem_bytes(p.rows_alloc);
-    const void* fn = philox ? (const void*)head_tc_kernel<true> : (const void*)head_tc_kernel<false>;
+    const void* fn = philox ? (const void*)head_tc_kernel<true, false>
+                            : (const void*)head_tc_kernel<false, false>;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
     void* args[] = {(void*)&tw, (void*)&th, (void*)&th64, (void*)&th128, (void*)&a};
@@ -920,6 +939,72 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     if (s != SBD_OK) return s;
   }
   return SBD_OK;
+}
+
+// y[T, N] = x[T, K] W[N, K]^T in bf16 with fp32 accumulation: the LM-head
+// kernel's main loop (W streamed once through the ring, x's rows from L2)
+// with a storing epilogue.
+sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y,
+                         cudaStream_t st) {
+  if (T == 0 || N == 0) return SBD_OK;
+  const int rows_alloc = T <= 16 ? 16 : ((T + 15) / 16) * 16;
+  CUtensorMap tw, tx, tx64, tx128;
+  sbd_status s;
+  {
+    const uint64_t dims[2] = {(uint64_t)K, (uint64_t)N};
+    const uint64_t strides[1] = {(uint64_t)K * 2};
+    const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)kBM};
+    s = encode_tensor_map(&tw, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)w, dims, strides, box,
+                          CU_TENSOR_MAP_SWIZZLE_128B);
+    if (s != SBD_OK) return s;
+  }
+  {
+    // rows of x past T (up to the MMA's multiple of 16) are read as zeros
+    const uint64_t dims[2] = {(uint64_t)K, (uint64_t)T};
+    const uint64_t strides[1] = {(uint64_t)K * 2};
+    const uint32_t box[2] = {(uint32_t)kBK, 16u};
+    s = encode_tensor_map(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)x, dims, strides, box,
+                          CU_TENSOR_MAP_SWIZZLE_128B);
+    if (s != SBD_OK) return s;
+    tx64 = tx;
+    tx128 = tx;
+    if (T >= 64) {
+      const uint32_t box64[2] = {(uint32_t)kBK, 64u};
+      s = encode_tensor_map(&tx64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)x, dims, strides,
+                            box64, CU_TENSOR_MAP_SWIZZLE_128B);
+      if (s != SBD_OK) return s;
+    }
+    if (T >= 128) {
+      const uint32_t box128[2] = {(uint32_t)kBK, 128u};
+      s = encode_tensor_map(&tx128, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)x, dims, strides,
+                            box128, CU_TENSOR_MAP_SWIZZLE_128B);
+      if (s != SBD_OK) return s;
+    }
+  }
+  HeadArgs a{};
+  a.err = device_error_word();
+  a.V = N;
+  a.H = K;
+  a.rows_alloc = rows_alloc;
+  a.n_tiles = (N + kBM - 1) / kBM;
+  a.h_big = SBD_HEAD_BIG_BOXES ? (T >= 128 ? 128 : (T >= 64 ? 64 : 16)) : 16;
+  a.ring_bytes = head_ring_bytes(rows_alloc);
+  const int n_acc_alloc = 2 * rows_alloc <= 512 ? 2 : 1;
+  uint32_t cols = 32;
+  while (cols < (uint32_t)(n_acc_alloc * rows_alloc)) cols <<= 1;
+  a.tmem_cols = cols;
+  a.tau = 0.f;
+  a.y = (__nv_bfloat16*)y;
+  a.linear_rows = T;
+  const size_t smem = head_smem_bytes(rows_alloc);
+  const void* fn = (const void*)head_tc_kernel<false, true>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel, linear)");
+  const int slots = num_sms() * SBD_HEAD_CTAS_PER_SM;
+  const int n_ctas = a.n_tiles < slots ? a.n_tiles : slots;
+  void* args[] = {(void*)&tw, (void*)&tx, (void*)&tx64, (void*)&tx128, (void*)&a};
+  return launch_pdl(fn, dim3(n_ctas), dim3(kHeadThreads), smem, st, args,
+                    "head_tc_kernel (linear) launch");
 }
 
 }  // namespace sbd

@@ -328,6 +328,30 @@ sbd_status sbd_head_entropy_sample_philox(const sbd_head_desc* desc, const void*
                    workspace_bytes, stream, &noise);
 }
 
+sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
+                      void* stream) {
+  if (!desc) return fail(SBD_ERR_INVALID_ARG, "desc is NULL");
+  if (desc->rows < 0 || desc->in_features < 1 || desc->out_features < 1)
+    return fail(SBD_ERR_INVALID_ARG, "bad sizes: rows=%d in_features=%d out_features=%d",
+                desc->rows, desc->in_features, desc->out_features);
+  if (desc->dtype != SBD_DTYPE_F32 && desc->dtype != SBD_DTYPE_BF16)
+    return fail(SBD_ERR_INVALID_ARG, "unknown dtype %d", desc->dtype);
+  if (desc->dtype != SBD_DTYPE_BF16) return fail(SBD_ERR_UNSUPPORTED, "sbd_linear is bf16 only");
+  if (desc->rows > 512) return fail(SBD_ERR_UNSUPPORTED, "rows %d > 512", desc->rows);
+  if (desc->in_features % 64 != 0)
+    return fail(SBD_ERR_UNSUPPORTED, "in_features %d is not a multiple of 64",
+                desc->in_features);
+  if (desc->rows == 0) return SBD_OK;
+  const void* ptrs[] = {x, w, y};
+  const char* names[] = {"x", "w", "y"};
+  for (int i = 0; i < 3; ++i) {
+    if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
+    if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
+  }
+  return sbd::linear_launch(desc->rows, desc->in_features, desc->out_features, x, w, y,
+                            (cudaStream_t)stream);
+}
+
 sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t vocab,
                              uint64_t seed, uint64_t offset, float* out, void* stream) {
   if (n_rows < 0 || vocab < 0)

@@ -57,6 +57,9 @@ size_t head_workspace_bytes(const HeadPlan& p);
 struct PhiloxNoise {
   uint64_t seed, offset;
 };
+// y[T, N] = x[T, K] W[N, K]^T, bf16 in and out, fp32 accumulation; T <= 512.
+sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y,
+                         cudaStream_t st);
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
                        float* confidence, int32_t* token, void* ws, cudaStream_t st,

@@ -180,6 +180,26 @@ def test_philox_calls_reject_bad_arguments(sbd):
     assert g(0, None, 10, 0, 0, None, None) == sbd.SBD_OK
 
 
+def test_linear_rejects_bad_arguments(sbd):
+    a = 1 << 20
+    f = sbd.lib.sbd_linear
+    L = sbd.LinearDesc
+    assert f(None, a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(-1, 64, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 0, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, 7)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_F32)), a, a, a, None) == sbd.SBD_ERR_UNSUPPORTED
+    assert f(ctypes.byref(L(513, 64, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == \
+        sbd.SBD_ERR_UNSUPPORTED
+    assert f(ctypes.byref(L(4, 96, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == \
+        sbd.SBD_ERR_UNSUPPORTED
+    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_BF16)), None, a, a, None) == \
+        sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_BF16)), a + 2, a, a, None) == \
+        sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(0, 64, 8, sbd.SBD_DTYPE_BF16)), None, None, None, None) == sbd.SBD_OK
+
+
 def test_binding_refuses_cpu_tensors(sbd):
     import torch
     x = torch.zeros(1, 4, 4, 64)

@@ -4,9 +4,11 @@ Every cell of the paper's printed slowdown and speedup tables (Sec. "Timing
 analysis", transcribed in tests/golden/roofline_tables.txt) must come out of
 the model rounded to the printed three decimals; plus the model's limits
 (time(1) ratios of 1, speedup equal to the NFE speedup when a block forward
-costs what a one-token forward does)."""
+costs what a one-token forward does); and the linear-layer GEMM of the
+measured forwards against its explicit triple sum."""
 import os
 
+import numpy as np
 import pytest
 
 import oracle
@@ -57,3 +59,13 @@ def test_gemm_roofline_regimes():
     assert t == pytest.approx((4096 + 4096 * 4096 + 4096) / c["bandwidth"])   # memory-bound
     t, f = oracle.roofline_gemm(8192, 8192, 8192)
     assert t == pytest.approx(2 * 8192 ** 3 / c["peak_flops"])                 # compute-bound
+
+
+def test_linear_is_the_explicit_triple_sum():
+    rng = np.random.default_rng(0)
+    x, w = rng.standard_normal((3, 5)), rng.standard_normal((4, 5))
+    y = oracle.linear(x, w)
+    for t in range(3):
+        for n in range(4):
+            assert y[t, n] == pytest.approx(sum(x[t, k] * w[n, k] for k in range(5)), abs=1e-12)
+    assert oracle.linear(np.zeros((2, 5)), w).shape == (2, 4)
