@@ -780,8 +780,10 @@ def run_speedup_tables(args):
     with the first k rows causal for 2k), the output projection and the
     SiLU-gated MLP; then the final norm and the LM head with entropy and
     Gumbel-max sample (sbd_head_entropy_sample) over the B n rows.
-    The projections are plain bf16 GEMMs (cuBLAS through torch.matmul): the
-    model's linear layers, outside the SBD step.  Every layer has its own
+    The projections are the GEMMs of the timing model: plain bf16 GEMMs by
+    cuBLAS (torch.matmul), or with --linear sbd by sbd_linear (the LM-head
+    kernel with a storing epilogue); the model's linear layers, outside the
+    SBD step.  Every layer has its own
     weights and KV cache, so nothing stays in L2 between layers; each forward
     is one CUDA graph, timed with CUDA events over `--steps` replays."""
     import torch
@@ -854,6 +856,14 @@ def run_speedup_tables(args):
                         calls.append(lambda kc=kc, vc=vc: sbd.sbd_block_attention(
                             qc, kc, vc, lens, kb, vb, out=attn_out, workspace=ws_a, stream=stream))
 
+                def linear(x_, w_, out_=None):
+                    # the layer's GEMM: cuBLAS (torch.matmul) or sbd_linear
+                    if args.linear == "sbd":
+                        return sbd.sbd_linear(x_, w_, out=out_, stream=stream)
+                    if out_ is None:
+                        return torch.matmul(x_, w_.t())
+                    return torch.matmul(x_, w_.t(), out=out_)
+
                 def rms(x):
                     xf = x.float()
                     return (xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + 1e-5)).bfloat16()
@@ -863,16 +873,16 @@ def run_speedup_tables(args):
                         x = x0
                         for li in range(NL):
                             Wl = layers_w[li]
-                            torch.matmul(rms(x), Wl["qkv"].t(), out=qkv_buf)
+                            linear(rms(x), Wl["qkv"], qkv_buf)
                             qc.copy_(q_v)                          # contiguous per-call layouts
                             kb.copy_(k_v.view(B, n, Hkv, D))
                             vb.copy_(v_v.view(B, n, Hkv, D))
                             calls[li]()
-                            o = torch.matmul(attn_out.view(T, Hq * D), Wl["o"].t())
+                            o = linear(attn_out.view(T, Hq * D), Wl["o"])
                             x = x + o
-                            gu = torch.matmul(rms(x), Wl["gu"].t())
+                            gu = linear(rms(x), Wl["gu"])
                             act = torch.nn.functional.silu(gu[:, :F]) * gu[:, F:]
-                            x = x + torch.matmul(act, Wl["down"].t())
+                            x = x + linear(act, Wl["down"])
                         hid.copy_(rms(x).view(B, n, H))
                         sbd.sbd_head_entropy_sample(hid, w_head, masked, gum, 1.0, ent, tok,
                                                     workspace=ws_h, stream=stream)
@@ -936,7 +946,8 @@ def run_speedup_tables(args):
         "config": {"workload": "speedup_tables", "model": "Llama-3.1-8B shapes, 32 layers",
                    "batches": list(SPEEDUP_BATCHES), "kv_lens": list(SPEEDUP_KV_LENS),
                    "block_sizes": list(SPEEDUP_KS), "nfe_speedups": list(SPEEDUP_NFE),
-                   "linear_layers": "cuBLAS bf16 GEMMs (torch.matmul)",
+                   "linear_layers": ("sbd_linear (tcgen05 LM-head kernel, storing epilogue)"
+                                     if args.linear == "sbd" else "cuBLAS bf16 GEMMs (torch.matmul)"),
                    "attention_and_head": "libsbd kernels"},
         "clocks": clocks,
         "tables": results,
@@ -962,6 +973,8 @@ def main():
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time eager launches, no CUDA graph")
+    ap.add_argument("--linear", choices=["cublas", "sbd"], default="cublas",
+                    help="GEMMs of the model's linear layers in --workload speedup_tables")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

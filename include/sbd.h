@@ -203,20 +203,29 @@ sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t voc
  *   x [rows, in_features]           bf16, row-major (device)
  *   w [out_features, in_features]   bf16, row-major, nn.Linear layout (device)
  *   y [rows, out_features]          bf16, row-major (device, written)
+ *   workspace                       sbd_linear_workspace_size(desc) bytes
+ *                                   (device, 16-byte aligned; may be NULL
+ *                                   when the size is 0)
  *
  * y is the fp32 sum over in_features of the bf16 products, rounded to
- * bf16 (round to nearest even).  All pointers 16-byte aligned, caller-owned;
- * no workspace.  Asynchronous on `stream`.
+ * bf16 (round to nearest even).  At up to 64 rows the in_features are cut
+ * into ranges summed in fp32 by a second kernel through the workspace, so
+ * that narrow layers still spread over all SMs.  All pointers 16-byte
+ * aligned, caller-owned.  Asynchronous on `stream`.
  * Supported: dtype bf16, 0 <= rows <= 512, in_features a positive multiple
- * of 64, out_features >= 1; SBD_ERR_UNSUPPORTED otherwise.
+ * of 64, out_features >= 1; SBD_ERR_UNSUPPORTED otherwise; a workspace
+ * smaller than needed gives SBD_ERR_WORKSPACE.
  * ---------------------------------------------------------------------- */
 typedef struct {
   int32_t rows, in_features, out_features;
   sbd_dtype dtype;
 } sbd_linear_desc;
 
+/* Bytes for the largest split the call may choose (the same on every
+ * device; 0 above 64 rows); 0 for an invalid descriptor. */
+size_t sbd_linear_workspace_size(const sbd_linear_desc* desc);
 sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
-                      void* stream);
+                      void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * No-allocation variant of sbd_head_entropy_sample.  The paper has no

@@ -49,6 +49,7 @@ EXPORTS = (
     "sbd_head_entropy_confidence_sample",
     "sbd_head_entropy_sample_philox",
     "sbd_gumbel_philox",
+    "sbd_linear_workspace_size",
     "sbd_linear",
     "sbd_eb_select",
     "sbd_select",
@@ -114,7 +115,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sbd_head_entropy_sample_philox.restype = ctypes.c_int
     lib.sbd_gumbel_philox.argtypes = [i32, vp, i32, u64, u64, vp, vp]
     lib.sbd_gumbel_philox.restype = ctypes.c_int
-    lib.sbd_linear.argtypes = [ctypes.POINTER(LinearDesc), vp, vp, vp, vp]
+    lib.sbd_linear_workspace_size.argtypes = [ctypes.POINTER(LinearDesc)]
+    lib.sbd_linear_workspace_size.restype = sz
+    lib.sbd_linear.argtypes = [ctypes.POINTER(LinearDesc), vp, vp, vp, vp, sz, vp]
     lib.sbd_linear.restype = ctypes.c_int
     lib.sbd_eb_select.argtypes = [i32, i32, vp, vp, f32, vp, vp, vp, vp]
     lib.sbd_eb_select.restype = ctypes.c_int
@@ -338,27 +341,43 @@ def sbd_gumbel_philox(row_ids, vocab: int, seed: int, offset: int, out=None, *, 
     return out
 
 
-def sbd_linear(x, w, out=None, *, stream=None):
-    """y = x W^T on the LM-head kernel: x [T, K] bf16, w [N, K] bf16
-    (nn.Linear layout), T <= 512, K a multiple of 64.  Returns out [T, N]
-    bf16."""
-    torch = _torch()
-    _need_cuda(x=x, w=w, out=out)
+def _linear_desc(x, w):
     if x.dim() != 2 or w.dim() != 2 or x.shape[1] != w.shape[1]:
         raise ValueError(f"shapes x {tuple(x.shape)} and w {tuple(w.shape)} do not match")
+    return LinearDesc(x.shape[0], x.shape[1], w.shape[0], _dtype_code(x))
+
+
+def sbd_linear(x, w, out=None, workspace=None, *, stream=None):
+    """y = x W^T on the LM-head kernel: x [T, K] bf16, w [N, K] bf16
+    (nn.Linear layout), T <= 512, K a multiple of 64.  Returns out [T, N]
+    bf16.  The workspace (fp32 partials when K is split at few rows) is
+    allocated here when not given."""
+    torch = _torch()
+    _need_cuda(x=x, w=w, out=out, workspace=workspace)
+    d = _linear_desc(x, w)
     if out is None:
         out = torch.empty((x.shape[0], w.shape[0]), dtype=x.dtype, device=x.device)
-    d = LinearDesc(x.shape[0], x.shape[1], w.shape[0], _dtype_code(x))
-    _check(lib.sbd_linear(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _stream(stream)))
+    need = lib.sbd_linear_workspace_size(ctypes.byref(d))
+    if workspace is None and need > 0:
+        workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib.sbd_linear(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _ptr(workspace), nbytes,
+                          _stream(stream)))
     return out
 
 
-def prepare_linear(x, w, out, *, stream=None) -> "Prepared":
+def prepare_linear(x, w, out, workspace=None, *, stream=None) -> "Prepared":
     """sbd_linear bound to fixed tensors (see Prepared)."""
-    _need_cuda(x=x, w=w, out=out)
-    d = LinearDesc(x.shape[0], x.shape[1], w.shape[0], _dtype_code(x))
-    args = (ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _stream(stream))
-    return Prepared(lib.sbd_linear, args, keep=(d, x, w, out))
+    torch = _torch()
+    _need_cuda(x=x, w=w, out=out, workspace=workspace)
+    d = _linear_desc(x, w)
+    need = lib.sbd_linear_workspace_size(ctypes.byref(d))
+    if workspace is None and need > 0:
+        workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    args = (ctypes.byref(d), _ptr(x), _ptr(w), _ptr(out), _ptr(workspace), nbytes,
+            _stream(stream))
+    return Prepared(lib.sbd_linear, args, keep=(d, x, w, out, workspace))
 
 
 def sbd_head_entropy_sample_noalloc(hidden, w, masked, gumbel, tau: float, entropy, token, *,

@@ -337,6 +337,8 @@ struct HeadArgs {
   int h_big;            // tallest hidden-row box encoded: 16, 64 or 128 rows
   __nv_bfloat16* y;     // kLinear: output [linear_rows, V]
   int linear_rows;      // kLinear: rows of x, all live
+  int ksplit;           // kLinear: K ranges per output tile (1: y written directly)
+  float* part_y;        // kLinear, ksplit > 1: fp32 partials [ksplit][linear_rows][V]
 };
 
 // kPhilox: the Gumbel noise is generated in the epilogue (philox.cuh)
@@ -394,9 +396,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   // than one box in 4-5: 160 rows 233 -> 219 us, 256 rows 255 -> 249 us;
   // four boxes in 2 stages slower than two in 4 at 60 rows.)
   const int b_box = n_eff * kBK * 2;
+  // kLinear at few rows: each output tile's K is cut into `ksplit` ranges,
+  // and the (tile, range) units are spread over the CTAs
+  const int ksplit = kLinear ? a.ksplit : 1;
+  const int n_units = a.n_tiles * ksplit;
   auto fits = [&](int bx, int n_st) { return ring_bytes / (bx * (kABytes + b_box)) >= n_st; };
   int boxes = SBD_HEAD_MAX_BOXES;
-  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || !fits(boxes, boxes > 2 ? 3 : 2)))
+  while (boxes > 1 &&
+         ((a.H / kBK) % (boxes * ksplit) != 0 || !fits(boxes, boxes > 2 ? 3 : 2)))
     boxes >>= 1;
   const int stage_bytes = boxes * (kABytes + b_box);     // [A boxes | B boxes]
   int stages = ring_bytes / stage_bytes;
@@ -427,7 +434,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
-  const int num_kb = a.H / (kBK * boxes);
+  const int num_kb = a.H / (kBK * boxes) / ksplit;   // stages per unit
 
   if (R > 0) {
     if (warp == 0) {
@@ -436,7 +443,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint64_t policy = l2_policy_evict_first();
         int it = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x) {
+        for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+          const int tile = u / ksplit, kb0 = (u % ksplit) * num_kb;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
             const int s = it % stages;
             const uint32_t ph = (it / stages) & 1;
@@ -447,7 +455,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
             uint8_t* st = ring + (size_t)s * stage_bytes;
             mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
             for (int x = 0; x < boxes; ++x) {
-              const int col = (kb * boxes + x) * kBK;
+              const int col = ((kb0 + kb) * boxes + x) * kBK;
 #if SBD_HEAD_EVICT_FIRST
               tma_load_2d_hint(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM, policy);
 #else
@@ -482,7 +490,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint32_t idesc_hi = idesc_bf16_f32(kBM, n_hi > 0 ? n_hi : 16);
         int it = 0, local = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < a.n_tiles; tile += gridDim.x, ++local) {
+        for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++local) {
           const int acc = n_acc == 2 ? (local & 1) : 0;
           const uint32_t use = (uint32_t)(n_acc == 2 ? (local >> 1) : local);
           if (!mbar_wait(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
@@ -521,7 +529,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const bool noisy = !kLinear && a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       int local = 0;
-      for (int tile = blockIdx.x; sub < n_sub && tile < a.n_tiles; tile += gridDim.x, ++local) {
+      for (int u = blockIdx.x; sub < n_sub && u < n_units; u += gridDim.x, ++local) {
+        const int tile = u / ksplit, ks = u % ksplit;
         const int acc = n_acc == 2 ? (local & 1) : 0;
         const uint32_t use = (uint32_t)(n_acc == 2 ? (local >> 1) : local);
         const int v0 = tile * kBM + quad * 32;
@@ -593,12 +602,20 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
           tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
           tc_wait_ld();
           if constexpr (kLinear) {
-            // y[c0 + j, v]: for each j the warp's lanes store 32 consecutive v
+            // y[c0 + j, v] (or its fp32 partial of K range ks): for each j the
+            // warp's lanes store 32 consecutive v
             if (valid) {
+              if (ksplit == 1) {
 #pragma unroll
-              for (int j = 0; j < 16; ++j)
-                if (c0 + j < R)
-                  a.y[(size_t)(c0 + j) * a.V + v] = __float2bfloat16_rn(__uint_as_float(r[j]));
+                for (int j = 0; j < 16; ++j)
+                  if (c0 + j < R)
+                    a.y[(size_t)(c0 + j) * a.V + v] = __float2bfloat16_rn(__uint_as_float(r[j]));
+              } else {
+                float* py = a.part_y + (size_t)ks * R * a.V;
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                  if (c0 + j < R) py[(size_t)(c0 + j) * a.V + v] = __uint_as_float(r[j]);
+              }
             }
           } else {
             float z[16];
@@ -790,6 +807,19 @@ size_t head_smem_bytes(int rows_alloc) {
   return 1024 + (size_t)head_scratch_bytes(rows_alloc) + head_ring_bytes(rows_alloc);
 }
 
+// y = the sum over K ranges of the fp32 partials of sbd_linear, in bf16.
+__global__ void __launch_bounds__(256)
+linear_reduce_kernel(const float* __restrict__ part, int ksplit, long long tn,
+                     __nv_bfloat16* __restrict__ y) {
+  grid_dependency_wait();
+  grid_dependents_launch();
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= tn) return;
+  float acc = 0.f;
+  for (int ks = 0; ks < ksplit; ++ks) acc += part[(size_t)ks * tn + i];
+  y[i] = __float2bfloat16_rn(acc);
+}
+
 }  // namespace
 
 namespace sbd {
@@ -888,6 +918,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.n_tiles = (p.V + kBM - 1) / kBM;
     a.y = nullptr;
     a.linear_rows = 0;
+    a.ksplit = 1;
+    a.part_y = nullptr;
     a.h_big = SBD_HEAD_BIG_BOXES ? (p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16)) : 16;
     a.ring_bytes = head_ring_bytes(p.rows_alloc);
     // tensor memory for two accumulators of the allocated width (one of it
@@ -944,10 +976,56 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
 // y[T, N] = x[T, K] W[N, K]^T in bf16 with fp32 accumulation: the LM-head
 // kernel's main loop (W streamed once through the ring, x's rows from L2)
 // with a storing epilogue.
-sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y,
+// The largest K split sbd_linear may use: powers of two up to 16, each K
+// range at least 4 column blocks long, at most 512 (tile, range) units and
+// at most 64 MB of fp32 partials.  A function of the shape only, so that
+// the workspace size does not depend on the device.
+static int linear_max_split(int T, int K, int N) {
+  const int kb64 = K / kBK, n_tiles = (N + kBM - 1) / kBM;
+  int ks = 1;
+  while (ks < 16 && kb64 % (2 * ks) == 0 && kb64 / (2 * ks) >= 4 &&
+         (long long)n_tiles * 2 * ks <= 512 &&
+         (long long)2 * ks * T * N * (long long)sizeof(float) <= (64ll << 20))
+    ks *= 2;
+  return ks;
+}
+
+int linear_ksplit(int T, int K, int N) {
+  // A time model per SM: a tile streams its 128 x K weights (~45 GB/s per
+  // SM at the HBM peak) or runs its 2 x 128 x n x K flops (~14.8 TFLOP/s
+  // per SM), whichever is longer; a unit of a split also writes its
+  // T x 128 fp32 partials, and the sum over ranges reads them all back in
+  // a second launch.  The split with the shortest modelled time wins.
+  const int max_ks = linear_max_split(T, K, N);
+  const int sms = num_sms() * SBD_HEAD_CTAS_PER_SM;
+  const int n_tiles = (N + kBM - 1) / kBM;
+  const double n_eff = T <= 16 ? 16.0 : (double)((T + 15) / 16 * 16);
+  const double t_mem = 128.0 * K * 2 / 45e3, t_mma = 2.0 * 128 * n_eff * K / 14.8e6;  // us
+  const double t_tile = t_mem > t_mma ? t_mem : t_mma;
+  const double t_part = (double)T * 128 * 4 / 45e3;
+  int best = 1;
+  double best_cost = (double)((n_tiles + sms - 1) / sms) * t_tile;
+  for (int ks = 2; ks <= max_ks; ks *= 2) {
+    const double waves = (double)((n_tiles * ks + sms - 1) / sms);
+    const double cost = waves * (t_tile / ks + t_part) + (double)ks * T * N * 4 / 6e6 + 2.0;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = ks;
+    }
+  }
+  return best;
+}
+
+size_t linear_workspace_bytes(int T, int K, int N) {
+  const int ks = linear_max_split(T, K, N);
+  return ks > 1 ? (size_t)ks * T * N * sizeof(float) : 0;
+}
+
+sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y, void* ws,
                          cudaStream_t st) {
   if (T == 0 || N == 0) return SBD_OK;
   const int rows_alloc = T <= 16 ? 16 : ((T + 15) / 16) * 16;
+  const int ksplit = linear_ksplit(T, K, N);
   CUtensorMap tw, tx, tx64, tx128;
   sbd_status s;
   {
@@ -996,15 +1074,26 @@ sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void
   a.tau = 0.f;
   a.y = (__nv_bfloat16*)y;
   a.linear_rows = T;
+  a.ksplit = ksplit;
+  a.part_y = (float*)ws;
   const size_t smem = head_smem_bytes(rows_alloc);
   const void* fn = (const void*)head_tc_kernel<false, true>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel, linear)");
   const int slots = num_sms() * SBD_HEAD_CTAS_PER_SM;
-  const int n_ctas = a.n_tiles < slots ? a.n_tiles : slots;
+  const int units = a.n_tiles * ksplit;
+  const int n_ctas = units < slots ? units : slots;
   void* args[] = {(void*)&tw, (void*)&tx, (void*)&tx64, (void*)&tx128, (void*)&a};
-  return launch_pdl(fn, dim3(n_ctas), dim3(kHeadThreads), smem, st, args,
-                    "head_tc_kernel (linear) launch");
+  s = launch_pdl(fn, dim3(n_ctas), dim3(kHeadThreads), smem, st, args,
+                 "head_tc_kernel (linear) launch");
+  if (s != SBD_OK || ksplit == 1) return s;
+  const float* part = (const float*)ws;
+  long long tn = (long long)T * N;
+  __nv_bfloat16* yb = (__nv_bfloat16*)y;
+  int ks = ksplit;
+  void* rargs[] = {(void*)&part, (void*)&ks, (void*)&tn, (void*)&yb};
+  return launch_pdl((const void*)linear_reduce_kernel, dim3((unsigned)((tn + 255) / 256)), dim3(256),
+                    0, st, rargs, "linear_reduce_kernel launch");
 }
 
 }  // namespace sbd

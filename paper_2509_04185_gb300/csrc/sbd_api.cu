@@ -328,8 +328,11 @@ sbd_status sbd_head_entropy_sample_philox(const sbd_head_desc* desc, const void*
                    workspace_bytes, stream, &noise);
 }
 
-sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
-                      void* stream) {
+}  // extern "C"
+
+namespace {
+
+sbd_status check_linear_desc(const sbd_linear_desc* desc) {
   if (!desc) return fail(SBD_ERR_INVALID_ARG, "desc is NULL");
   if (desc->rows < 0 || desc->in_features < 1 || desc->out_features < 1)
     return fail(SBD_ERR_INVALID_ARG, "bad sizes: rows=%d in_features=%d out_features=%d",
@@ -341,6 +344,22 @@ sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w,
   if (desc->in_features % 64 != 0)
     return fail(SBD_ERR_UNSUPPORTED, "in_features %d is not a multiple of 64",
                 desc->in_features);
+  return SBD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t sbd_linear_workspace_size(const sbd_linear_desc* desc) {
+  if (check_linear_desc(desc) != SBD_OK) return 0;
+  return sbd::linear_workspace_bytes(desc->rows, desc->in_features, desc->out_features);
+}
+
+sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
+                      void* workspace, size_t workspace_bytes, void* stream) {
+  sbd_status s = check_linear_desc(desc);
+  if (s != SBD_OK) return s;
   if (desc->rows == 0) return SBD_OK;
   const void* ptrs[] = {x, w, y};
   const char* names[] = {"x", "w", "y"};
@@ -348,8 +367,15 @@ sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w,
     if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
     if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
   }
+  const size_t need = sbd::linear_workspace_bytes(desc->rows, desc->in_features,
+                                                  desc->out_features);
+  if (need > 0 && (!workspace || workspace_bytes < need))
+    return fail(SBD_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
+                workspace ? workspace_bytes : (size_t)0);
+  if (need > 0 && !aligned16(workspace))
+    return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
   return sbd::linear_launch(desc->rows, desc->in_features, desc->out_features, x, w, y,
-                            (cudaStream_t)stream);
+                            workspace, (cudaStream_t)stream);
 }
 
 sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t vocab,

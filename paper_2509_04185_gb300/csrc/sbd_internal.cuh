@@ -58,7 +58,11 @@ struct PhiloxNoise {
   uint64_t seed, offset;
 };
 // y[T, N] = x[T, K] W[N, K]^T, bf16 in and out, fp32 accumulation; T <= 512.
-sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y,
+// At few rows K is split over CTAs (linear_ksplit ranges), with fp32 partials
+// in the workspace (linear_workspace_bytes) summed by a second kernel.
+int linear_ksplit(int T, int K, int N);
+size_t linear_workspace_bytes(int T, int K, int N);
+sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void* y, void* ws,
                          cudaStream_t st);
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,

@@ -184,20 +184,28 @@ def test_linear_rejects_bad_arguments(sbd):
     a = 1 << 20
     f = sbd.lib.sbd_linear
     L = sbd.LinearDesc
-    assert f(None, a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(-1, 64, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(4, 0, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(4, 64, 8, 7)), a, a, a, None) == sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_F32)), a, a, a, None) == sbd.SBD_ERR_UNSUPPORTED
-    assert f(ctypes.byref(L(513, 64, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == \
+    bf = sbd.SBD_DTYPE_BF16
+    big = 1 << 30
+    assert f(None, a, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(-1, 64, 8, bf)), a, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 0, 8, bf)), a, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, 7)), a, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_F32)), a, a, a, a, big, None) == \
         sbd.SBD_ERR_UNSUPPORTED
-    assert f(ctypes.byref(L(4, 96, 8, sbd.SBD_DTYPE_BF16)), a, a, a, None) == \
-        sbd.SBD_ERR_UNSUPPORTED
-    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_BF16)), None, a, a, None) == \
-        sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(4, 64, 8, sbd.SBD_DTYPE_BF16)), a + 2, a, a, None) == \
-        sbd.SBD_ERR_INVALID_ARG
-    assert f(ctypes.byref(L(0, 64, 8, sbd.SBD_DTYPE_BF16)), None, None, None, None) == sbd.SBD_OK
+    assert f(ctypes.byref(L(513, 64, 8, bf)), a, a, a, a, big, None) == sbd.SBD_ERR_UNSUPPORTED
+    assert f(ctypes.byref(L(4, 96, 8, bf)), a, a, a, a, big, None) == sbd.SBD_ERR_UNSUPPORTED
+    assert f(ctypes.byref(L(4, 64, 8, bf)), None, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(4, 64, 8, bf)), a + 2, a, a, a, big, None) == sbd.SBD_ERR_INVALID_ARG
+    assert f(ctypes.byref(L(0, 64, 8, bf)), None, None, None, None, 0, None) == sbd.SBD_OK
+    size = sbd.lib.sbd_linear_workspace_size
+    assert size(None) == 0 and size(ctypes.byref(L(513, 64, 8, bf))) == 0
+    # a narrow layer at few rows splits K: fp32 partials need a workspace
+    d = L(16, 4096, 4096, bf)
+    need = size(ctypes.byref(d))
+    assert need == 16 * 16 * 4096 * 4        # sized for the largest split (16 ranges)
+    assert f(ctypes.byref(d), a, a, a, None, 0, None) == sbd.SBD_ERR_WORKSPACE
+    assert f(ctypes.byref(d), a, a, a, a, need - 1, None) == sbd.SBD_ERR_WORKSPACE
+    assert size(ctypes.byref(L(512, 4096, 65536, bf))) == 0     # 512 tiles: never split
 
 
 def test_binding_refuses_cpu_tensors(sbd):

@@ -23,7 +23,9 @@ def _bf16(rng, shape, scale):
 @pytest.mark.parametrize("T,K,N", [(1, 4096, 6144), (5, 64, 1), (16, 256, 129), (17, 256, 1000),
                                    (64, 4096, 128), (100, 512, 777), (128, 1024, 2048),
                                    (200, 256, 300), (256, 4096, 4096), (300, 128, 129),
-                                   (512, 256, 1000)])
+                                   (512, 256, 1000),
+                                   # few rows, narrow layers: K split over CTAs
+                                   (16, 4096, 4096), (2, 14336, 512), (64, 1024, 300)])
 def test_matches_fp64_product(sbd, T, K, N):
     import torch
     rng = np.random.default_rng(T * 7 + N)
