@@ -22,6 +22,11 @@
 //   head_combine_kernel  merges the per-CTA statistics of each row into the
 //                        entropy (nats), the token and, when asked for, the
 //                        confidence max_v p_v = 1 / S.
+//
+// head_tc_kernel also serves sbd_linear (y = x W^T, a template switch): the
+// same main loop over all rows of x, an epilogue that stores the
+// accumulators (or, with K split over CTAs at few rows, fp32 partials that
+// linear_reduce_kernel sums).
 #include <math.h>
 
 #include "philox.cuh"
