@@ -583,9 +583,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     grid_dependents_launch();
     // ------------------------------------------------ epilogue
-    // Row sums over the group, in a fixed order.  The first barrier lets the
-    // group finish reading the last pair's maxima before the buffer is reused.
-    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
+    // Row sums over the group, in a fixed order.  They reuse the buffer of
+    // the maxima, whose slots of every group they overlap, and a slower
+    // group may still be reading the last pair's maxima: all softmax warps
+    // pass one barrier (id 5; the groups use 1-4) before any sum is written.
+    asm volatile("bar.sync 5, %0;" ::"n"(kSoftWarps * 32) : "memory");
     red_l[sw * 32 + lane] = l;
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
     float lsum = 0.f;
