@@ -474,39 +474,51 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
 }
 
 // Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.  One CTA per
-// (packed row, KV head, sequence); thread d owns output element d.
+// (packed row, KV head, sequence); thread d owns output element d.  The
+// kernel is latency-bound: every thread issues the loads of up to 32 splits
+// (their log-sum-exps, broadcast within a warp, and its own column of their
+// outputs) before using any of them, so that one memory round trip covers
+// them, and merges each group of 32 online.
 template <typename OutT>
 __global__ void __launch_bounds__(128)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
                     OutT* __restrict__ out, int k, int Hq, int Hkv, int G, int M, int D,
                     int splits) {
-  __shared__ float w_s[64];
-  __shared__ float inv_sum;
+  constexpr int kGroup = 32;
   grid_dependency_wait();
   const int r = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
-  const size_t pair = (size_t)b * Hkv + hkv;
-  const float* lse = part_lse + pair * splits * M;
-  if (threadIdx.x < 32) {
-    const int lane = threadIdx.x;
-    float mx = -INFINITY;
-    for (int s = lane; s < splits; s += 32) mx = fmaxf(mx, lse[(size_t)s * M + r]);
-    mx = warp_max(mx);
-    float sum = 0.f;
-    for (int s = lane; s < splits; s += 32) {
-      const float wt = (mx == -INFINITY) ? 0.f : exp2f(lse[(size_t)s * M + r] - mx);
-      w_s[s] = wt;
-      sum += wt;
-    }
-    sum = warp_sum(sum);
-    if (lane == 0) inv_sum = sum > 0.f ? 1.f / sum : 0.f;
-  }
-  __syncthreads();
   const int d = threadIdx.x;
   if (d >= D) return;
+  const size_t pair = (size_t)b * Hkv + hkv;
+  const float* lse = part_lse + pair * splits * M + r;
   const float* po = part_o + (pair * splits * M + r) * D + d;
-  float acc = 0.f;
-  for (int s = 0; s < splits; ++s) acc += w_s[s] * po[(size_t)s * M * D];
-  acc *= inv_sum;
+  float mx = -INFINITY, sum = 0.f, acc = 0.f;
+  for (int s0 = 0; s0 < splits; s0 += kGroup) {
+    float l[kGroup], v[kGroup];
+#pragma unroll
+    for (int e = 0; e < kGroup; ++e) {
+      const int s = s0 + e;
+      l[e] = s < splits ? lse[(size_t)s * M] : -INFINITY;
+      v[e] = s < splits ? po[(size_t)s * M * D] : 0.f;
+    }
+    float gm = l[0];
+#pragma unroll
+    for (int e = 1; e < kGroup; ++e) gm = fmaxf(gm, l[e]);
+    if (gm == -INFINITY) continue;               // every split of the group is empty
+    if (gm > mx) {
+      const float c = exp2f(mx - gm);            // 0 while mx = -inf
+      sum *= c;
+      acc *= c;
+      mx = gm;
+    }
+#pragma unroll
+    for (int e = 0; e < kGroup; ++e) {
+      const float wt = exp2f(l[e] - mx);
+      sum += wt;
+      if (wt > 0.f) acc = fmaf(wt, v[e], acc);
+    }
+  }
+  acc = sum > 0.f ? acc / sum : 0.f;
   const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + d;
   if constexpr (sizeof(OutT) == 2)
     out[o] = __float2bfloat16_rn(acc);

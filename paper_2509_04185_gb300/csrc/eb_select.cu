@@ -39,24 +39,31 @@ select_kernel(int B, int k, const float* __restrict__ entropy,
   const int b = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   if (b >= B) return;
 
+  // All loads are issued before any is used (the kernel is latency-bound);
+  // the values of unmasked lanes are not used.
   const bool in_block = lane < k;
-  const bool is_masked = in_block && masked[(size_t)b * k + lane] != 0;
+  const size_t at = (size_t)b * k + lane;
+  const uint8_t m_raw = in_block ? masked[at] : (uint8_t)0;
+  const float h_raw = in_block ? entropy[at] : 0.f;
+  const float c_raw = (in_block && !kByEntropy) ? confidence[at] : 0.f;
+  int tok = in_block ? token[at] : 0;
+  const bool is_masked = m_raw != 0;
   float h = INFINITY;      // entropy
   float key = INFINITY;    // sort key, ascending
   if (is_masked) {
-    h = entropy[(size_t)b * k + lane];
+    h = h_raw;
     if (kByEntropy) {
       key = isnan(h) ? INFINITY : h;         // a NaN sorts last among masked
       h = key;
     } else {
-      const float c = confidence[(size_t)b * k + lane];
-      key = isnan(c) ? INFINITY : -c;        // confidence descending
+      key = isnan(c_raw) ? INFINITY : -c_raw;   // confidence descending
     }
   }
   // Unmasked lanes sort after every masked one (position key offset by 32).
   int key_pos = is_masked ? lane : lane + 32;
 
-  // Bitonic sort of 32 (key, position) pairs, ascending; the entropy rides along.
+  // Bitonic sort of 32 (key, position) pairs, ascending; the entropy and the
+  // sampled token ride along.
 #pragma unroll
   for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
@@ -64,6 +71,7 @@ select_kernel(int B, int k, const float* __restrict__ entropy,
       const float ok = __shfl_xor_sync(0xffffffffu, key, stride);
       const int op = __shfl_xor_sync(0xffffffffu, key_pos, stride);
       const float oh = kByEntropy ? ok : __shfl_xor_sync(0xffffffffu, h, stride);
+      const int ot = __shfl_xor_sync(0xffffffffu, tok, stride);
       const bool ascending = (lane & size) == 0 || size == 32;
       const bool lower = (lane & stride) == 0;
       const bool other_less = key_less(ok, op, key, key_pos);
@@ -72,6 +80,7 @@ select_kernel(int B, int k, const float* __restrict__ entropy,
         key = ok;
         key_pos = op;
         h = oh;
+        tok = ot;
       }
     }
   }
@@ -117,7 +126,7 @@ select_kernel(int B, int k, const float* __restrict__ entropy,
   if (lane < s) {
     const int pos = key_pos;                       // original block position
     const size_t o = (size_t)b * k + pos;
-    block_tokens[o] = token[o];
+    block_tokens[o] = tok;
     masked[o] = 0;
   }
   if (lane == 0 && n_unmasked) n_unmasked[b] = s;

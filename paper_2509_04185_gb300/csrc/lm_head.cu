@@ -729,27 +729,47 @@ head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
 
 // ------------------------------------------------------------ combine
 // One warp per masked row: merge the per-CTA statistics, then
-// H = ln 2 * (log2 S - T / S)  (nats) and the winning token.
+// H = ln 2 * (log2 S - T / S)  (nats) and the winning token.  Latency-bound:
+// the row count, the row map and up to 256 CTAs' statistics (8 per lane) are
+// all requested before any of them is used.
 __global__ void __launch_bounds__(128)
 head_combine_kernel(const float4* __restrict__ part_msTb, const int32_t* __restrict__ part_idx,
                     int n_parts, int rows_alloc, const int32_t* __restrict__ row_map,
                     const int32_t* __restrict__ n_rows, float* __restrict__ entropy,
                     int32_t* __restrict__ token, float* __restrict__ confidence) {
+  constexpr int kPerLane = 8;
   grid_dependency_wait();
   const int r = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (r >= *n_rows) return;
+  if (r >= rows_alloc) return;
+  const int rows = *n_rows;
+  const int row = row_map[r];        // read before the check: r < rows_alloc
   RowStats s = rowstats_empty();
-  for (int c = lane; c < n_parts; c += 32) {
-    const float4 v = part_msTb[(size_t)c * rows_alloc + r];
-    RowStats o;
-    o.m = v.x;
-    o.S = v.y;
-    o.T = v.z;
-    o.best = v.w;
-    o.idx = part_idx[(size_t)c * rows_alloc + r];
-    s = rowstats_merge(s, o);
+  for (int c0 = 0; c0 < n_parts; c0 += 32 * kPerLane) {
+    float4 v[kPerLane];
+    int id[kPerLane];
+#pragma unroll
+    for (int e = 0; e < kPerLane; ++e) {
+      const int c = c0 + e * 32 + lane;
+      if (c < n_parts) {
+        v[e] = part_msTb[(size_t)c * rows_alloc + r];
+        id[e] = part_idx[(size_t)c * rows_alloc + r];
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < kPerLane; ++e) {
+      if (c0 + e * 32 + lane < n_parts) {
+        RowStats o;
+        o.m = v[e].x;
+        o.S = v[e].y;
+        o.T = v[e].z;
+        o.best = v[e].w;
+        o.idx = id[e];
+        s = rowstats_merge(s, o);
+      }
+    }
   }
+  if (r >= rows) return;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     RowStats t;
@@ -761,7 +781,6 @@ head_combine_kernel(const float4* __restrict__ part_msTb, const int32_t* __restr
     s = rowstats_merge(s, t);
   }
   if (lane == 0) {
-    const int row = row_map[r];
     entropy[row] = kLn2 * (log2f(s.S) - s.T / s.S);
     token[row] = s.idx;
     // the largest probability is the max term's: 2^0 / S
