@@ -168,6 +168,14 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
       tma_prefetch_desc(&tmap_k);
       tma_prefetch_desc(&tmap_v);
     }
+    // The split that ends with the block tile asks for the block rows' keys
+    // and values now (into L2); it copies them after its cache tiles.
+    if (t_end == n_tiles)
+      for (int c = lane; c < 2 * a.k * (D / 64); c += 32) {
+        const int row = c / (2 * (D / 64)), part = c % (2 * (D / 64));
+        const __nv_bfloat16* src = part < D / 64 ? a.kb : a.vb;
+        prefetch_l2(src + (((size_t)b * a.k + row) * a.Hkv + hkv) * D + (part % (D / 64)) * 64);
+      }
     int it = 0;
     for (int t = t_begin; t < t_end; ++t, ++it) {
       const int stage = it % kStages;
@@ -186,32 +194,47 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
           }
         }
       } else {
-        // Block keys/values: rows j < k copied, rows k..63 zero.
-        const int chunks_per_row = D / 8;                       // 16-byte chunks
-        for (int c = lane; c < kTileKeys * chunks_per_row; c += 32) {
-          const int j = c / chunks_per_row, cc = c % chunks_per_row;
-          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-          if (j < a.k) {
-            const size_t off = (((size_t)b * a.k + j) * a.Hkv + hkv) * D + cc * 8;
-            kv = *reinterpret_cast<const uint4*>(a.kb + off);
-            vv = *reinterpret_cast<const uint4*>(a.vb + off);
-            if (a.kc_app && j < a.n_causal && len + a.n_causal <= a.Lmax) {
+        // Block keys/values: rows j < k copied, rows k..63 zero.  Each batch
+        // issues all of a lane's loads before its stores (shared stores are
+        // volatile asm), so that it costs one memory round trip.
+        constexpr int chunks_per_row = D / 8;                   // 16-byte chunks
+        constexpr int kBatch = 8;                               // chunks per lane per batch
+        const int n_valid = a.k * chunks_per_row;               // chunks of rows < k
+        for (int c0 = 0; c0 < kTileKeys * chunks_per_row; c0 += 32 * kBatch) {
+          uint4 kv[kBatch], vv[kBatch];
+#pragma unroll
+          for (int e = 0; e < kBatch; ++e) {
+            const int c = c0 + e * 32 + lane;
+            kv[e] = make_uint4(0, 0, 0, 0);
+            vv[e] = make_uint4(0, 0, 0, 0);
+            if (c < n_valid) {
+              const size_t off =
+                  (((size_t)b * a.k + c / chunks_per_row) * a.Hkv + hkv) * D + (c % chunks_per_row) * 8;
+              kv[e] = *reinterpret_cast<const uint4*>(a.kb + off);
+              vv[e] = *reinterpret_cast<const uint4*>(a.vb + off);
+            }
+          }
+#pragma unroll
+          for (int e = 0; e < kBatch; ++e) {
+            const int c = c0 + e * 32 + lane;
+            const int j = c / chunks_per_row, cc = c % chunks_per_row;
+            if (a.kc_app && c < n_valid && j < a.n_causal && len + a.n_causal <= a.Lmax) {
               // a causal row enters the cache (positions >= len are read by
               // no split of this call, or masked and zeroed where they are)
               const size_t dst = (((size_t)b * a.Lmax + len + j) * a.Hkv + hkv) * D + cc * 8;
-              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv;
-              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv;
+              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv[e];
+              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv[e];
             }
+            const int h = cc / 8, c8 = cc % 8;
+            const uint32_t ka = swz(kbase + h * kSubBytes, j, c8);
+            const uint32_t va = swz(vbase + h * kSubBytes, j, c8);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(ka), "r"(kv[e].x),
+                         "r"(kv[e].y), "r"(kv[e].z), "r"(kv[e].w)
+                         : "memory");
+            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(va), "r"(vv[e].x),
+                         "r"(vv[e].y), "r"(vv[e].z), "r"(vv[e].w)
+                         : "memory");
           }
-          const int h = cc / 8, c8 = cc % 8;
-          const uint32_t ka = swz(kbase + h * kSubBytes, j, c8);
-          const uint32_t va = swz(vbase + h * kSubBytes, j, c8);
-          asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(ka), "r"(kv.x), "r"(kv.y),
-                       "r"(kv.z), "r"(kv.w)
-                       : "memory");
-          asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(va), "r"(vv.x), "r"(vv.y),
-                       "r"(vv.z), "r"(vv.w)
-                       : "memory");
         }
         if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
           record_error(a.err, SBD_DEVERR_CACHE_LEN);
@@ -474,11 +497,11 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
 }
 
 // Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.  One CTA per
-// (packed row, KV head, sequence); thread d owns output element d.  The
-// kernel is latency-bound: every thread issues the loads of up to 32 splits
-// (their log-sum-exps, broadcast within a warp, and its own column of their
-// outputs) before using any of them, so that one memory round trip covers
-// them, and merges each group of 32 online.
+// (packed row, KV head, sequence); thread d owns output element d (D is 64
+// or 128, so whole warps take part).  The kernel is latency-bound: for each
+// group of 32 splits a thread requests its column of all of them, and lane s
+// the log-sum-exp of split s (shared through shuffles), before any is used,
+// so that one memory round trip covers the group; groups merge online.
 template <typename OutT>
 __global__ void __launch_bounds__(128)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
@@ -487,23 +510,18 @@ attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ 
   constexpr int kGroup = 32;
   grid_dependency_wait();
   const int r = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
-  const int d = threadIdx.x;
+  const int d = threadIdx.x, lane = threadIdx.x & 31;
   if (d >= D) return;
   const size_t pair = (size_t)b * Hkv + hkv;
   const float* lse = part_lse + pair * splits * M + r;
   const float* po = part_o + (pair * splits * M + r) * D + d;
   float mx = -INFINITY, sum = 0.f, acc = 0.f;
   for (int s0 = 0; s0 < splits; s0 += kGroup) {
-    float l[kGroup], v[kGroup];
+    const float l_lane = s0 + lane < splits ? lse[(size_t)(s0 + lane) * M] : -INFINITY;
+    float v[kGroup];
 #pragma unroll
-    for (int e = 0; e < kGroup; ++e) {
-      const int s = s0 + e;
-      l[e] = s < splits ? lse[(size_t)s * M] : -INFINITY;
-      v[e] = s < splits ? po[(size_t)s * M * D] : 0.f;
-    }
-    float gm = l[0];
-#pragma unroll
-    for (int e = 1; e < kGroup; ++e) gm = fmaxf(gm, l[e]);
+    for (int e = 0; e < kGroup; ++e) v[e] = s0 + e < splits ? po[(size_t)(s0 + e) * M * D] : 0.f;
+    const float gm = warp_max(l_lane);
     if (gm == -INFINITY) continue;               // every split of the group is empty
     if (gm > mx) {
       const float c = exp2f(mx - gm);            // 0 while mx = -inf
@@ -513,7 +531,7 @@ attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ 
     }
 #pragma unroll
     for (int e = 0; e < kGroup; ++e) {
-      const float wt = exp2f(l[e] - mx);
+      const float wt = exp2f(__shfl_sync(0xffffffffu, l_lane, e) - mx);
       sum += wt;
       if (wt > 0.f) acc = fmaf(wt, v[e], acc);
     }

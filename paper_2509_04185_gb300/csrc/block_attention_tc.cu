@@ -293,6 +293,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     };
     if (lane == 0)
       for (int t = t_begin + kStages; t < t_begin + kStages + SBD_ATTN_L2_AHEAD; ++t) prefetch(t);
+    // The split that ends with the block tile asks for the block rows' keys
+    // and values now (into L2); it copies them after its cache tiles.
+    if (t_end == n_tiles)
+      for (int c = lane; c < 2 * a.k * (D / 64); c += 32) {
+        const int row = c / (2 * (D / 64)), part = c % (2 * (D / 64));
+        const __nv_bfloat16* src = part < D / 64 ? a.kb : a.vb;
+        prefetch_l2(src + (((size_t)b * a.k + row) * a.Hkv + hkv) * D + (part % (D / 64)) * 64);
+      }
     for (int j = 0; j < n; ++j) {
       const int t = t_begin + j;
       const int stage = j % kStages;
@@ -330,23 +338,38 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       } else {
         // Block keys/values (not cached): rows j < k copied, rows k..63 zero.
-        for (int c = lane; c < kTileKeys * kSub * 8; c += 32) {
-          const int row = c / (kSub * 8), cc = c % (kSub * 8);
-          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-          if (row < a.k) {
-            const size_t off = (((size_t)b * a.k + row) * a.Hkv + hkv) * D + cc * 8;
-            kv = *reinterpret_cast<const uint4*>(a.kb + off);
-            vv = *reinterpret_cast<const uint4*>(a.vb + off);
-            if (a.kc_app && row < a.n_causal && len + a.n_causal <= a.Lmax) {
+        // Each batch issues all of a lane's loads before its stores (shared
+        // stores are volatile asm), so that it costs one memory round trip.
+        constexpr int kCpr = kSub * 8;                 // 16-byte chunks per row
+        constexpr int kBatch = 8;                      // chunks per lane per batch
+        const int n_valid = a.k * kCpr;                // chunks of rows < k
+        for (int c0 = 0; c0 < kTileKeys * kCpr; c0 += 32 * kBatch) {
+          uint4 kv[kBatch], vv[kBatch];
+#pragma unroll
+          for (int e = 0; e < kBatch; ++e) {
+            const int c = c0 + e * 32 + lane;
+            kv[e] = make_uint4(0, 0, 0, 0);
+            vv[e] = make_uint4(0, 0, 0, 0);
+            if (c < n_valid) {
+              const size_t off = (((size_t)b * a.k + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
+              kv[e] = *reinterpret_cast<const uint4*>(a.kb + off);
+              vv[e] = *reinterpret_cast<const uint4*>(a.vb + off);
+            }
+          }
+#pragma unroll
+          for (int e = 0; e < kBatch; ++e) {
+            const int c = c0 + e * 32 + lane;
+            const int row = c / kCpr, cc = c % kCpr;
+            if (a.kc_app && c < n_valid && row < a.n_causal && len + a.n_causal <= a.Lmax) {
               // a causal row enters the cache (positions >= len are read by
               // no split of this call, or masked and zeroed where they are)
               const size_t dst = (((size_t)b * a.Lmax + len + row) * a.Hkv + hkv) * D + cc * 8;
-              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv;
-              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv;
+              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv[e];
+              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv[e];
             }
+            st_shared_v4(swz(k_chunk(j, cc / 8), row, cc % 8), kv[e]);
+            st_shared_v4(swz(v_chunk(j, cc / 8), row, cc % 8), vv[e]);
           }
-          st_shared_v4(swz(k_chunk(j, cc / 8), row, cc % 8), kv);
-          st_shared_v4(swz(v_chunk(j, cc / 8), row, cc % 8), vv);
         }
         if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
           record_error(a.err, SBD_DEVERR_CACHE_LEN);
