@@ -20,8 +20,8 @@
 // with 128-key pairs).  The two tiles of a pair sit back to back in every
 // 128-byte sub-tile of the ring, so that they form one 128-row operand.
 //
-// Warp roles: warp 0 streams K/V tiles with TMA (a ring of 3 pairs) and
-// copies the k block keys/values as the last tile of the last split; warp 1
+// Warp roles: warp 0 streams K/V tiles with TMA (a ring of 3 pairs), the k
+// block keys/values included (the last tile of the last split); warp 1
 // owns the tensor memory and one thread issues the MMAs, computing S_{q+1}
 // while the softmax of pair q runs; warps 2-9 are the softmax, two per TMEM
 // lane quadrant (and, with 64 packed rows or fewer, each row copied to a
@@ -187,7 +187,9 @@ struct TcArgs {
 template <int D, int R>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
-               const __grid_constant__ CUtensorMap tmap_v, const TcArgs a) {
+               const __grid_constant__ CUtensorMap tmap_v,
+               const __grid_constant__ CUtensorMap tmap_kb,
+               const __grid_constant__ CUtensorMap tmap_vb, const TcArgs a) {
   constexpr int kSub = D / 64;                     // 128-B column sub-tiles of a key row
   constexpr int kQBytes = kRows * 128;             // one Q (or P) sub-tile: 16 KB
   constexpr int kKVSub = kTileKeys * 128;          // one tile's K or V sub-tile: 8 KB
@@ -282,6 +284,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     if (lane == 0) {
       tma_prefetch_desc(&tmap_k);
       tma_prefetch_desc(&tmap_v);
+      if (t_end == n_tiles) {
+        tma_prefetch_desc(&tmap_kb);
+        tma_prefetch_desc(&tmap_vb);
+      }
     }
     auto prefetch = [&](int t) {
       if (SBD_ATTN_L2_AHEAD > 0 && t < t_end && t < n_cache_tiles) {
@@ -293,14 +299,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     };
     if (lane == 0)
       for (int t = t_begin + kStages; t < t_begin + kStages + SBD_ATTN_L2_AHEAD; ++t) prefetch(t);
-    // The split that ends with the block tile asks for the block rows' keys
-    // and values now (into L2); it copies them after its cache tiles.
-    if (t_end == n_tiles)
-      for (int c = lane; c < 2 * a.k * (D / 64); c += 32) {
-        const int row = c / (2 * (D / 64)), part = c % (2 * (D / 64));
-        const __nv_bfloat16* src = part < D / 64 ? a.kb : a.vb;
-        prefetch_l2(src + (((size_t)b * a.k + row) * a.Hkv + hkv) * D + (part % (D / 64)) * 64);
-      }
     for (int j = 0; j < n; ++j) {
       const int t = t_begin + j;
       const int stage = j % kStages;
@@ -337,45 +335,54 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           if (lane == 0) mbar_arrive(&kv_full[stage]);
         }
       } else {
-        // Block keys/values (not cached): rows j < k copied, rows k..63 zero.
-        // Each batch issues all of a lane's loads before its stores (shared
-        // stores are volatile asm), so that it costs one memory round trip.
-        constexpr int kCpr = kSub * 8;                 // 16-byte chunks per row
-        constexpr int kBatch = 8;                      // chunks per lane per batch
-        const int n_valid = a.k * kCpr;                // chunks of rows < k
-        for (int c0 = 0; c0 < kTileKeys * kCpr; c0 += 32 * kBatch) {
-          uint4 kv[kBatch], vv[kBatch];
-#pragma unroll
-          for (int e = 0; e < kBatch; ++e) {
-            const int c = c0 + e * 32 + lane;
-            kv[e] = make_uint4(0, 0, 0, 0);
-            vv[e] = make_uint4(0, 0, 0, 0);
-            if (c < n_valid) {
-              const size_t off = (((size_t)b * a.k + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
-              kv[e] = *reinterpret_cast<const uint4*>(a.kb + off);
-              vv[e] = *reinterpret_cast<const uint4*>(a.vb + off);
-            }
-          }
-#pragma unroll
-          for (int e = 0; e < kBatch; ++e) {
-            const int c = c0 + e * 32 + lane;
-            const int row = c / kCpr, cc = c % kCpr;
-            if (a.kc_app && c < n_valid && row < a.n_causal && len + a.n_causal <= a.Lmax) {
-              // a causal row enters the cache (positions >= len are read by
-              // no split of this call, or masked and zeroed where they are)
-              const size_t dst = (((size_t)b * a.Lmax + len + row) * a.Hkv + hkv) * D + cc * 8;
-              *reinterpret_cast<uint4*>(a.kc_app + dst) = kv[e];
-              *reinterpret_cast<uint4*>(a.vc_app + dst) = vv[e];
-            }
-            st_shared_v4(swz(k_chunk(j, cc / 8), row, cc % 8), kv[e]);
-            st_shared_v4(swz(v_chunk(j, cc / 8), row, cc % 8), vv[e]);
+        // Block keys/values (not cached): one TMA box per sub-tile from the
+        // [B, k, Hkv, D] block tensors, like a cache tile; rows k..63 lie
+        // outside those tensors and arrive as zeros.
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&kv_full[stage], 2 * kSub * kKVSub);
+          for (int h = 0; h < kSub; ++h) {
+            tma_load_4d(smem_raw + (k_chunk(j, h) - smem_u32(smem_raw)), &tmap_kb, &kv_full[stage],
+                        64 * h, hkv, 0, b);
+            tma_load_4d(smem_raw + (v_chunk(j, h) - smem_u32(smem_raw)), &tmap_vb, &kv_full[stage],
+                        64 * h, hkv, 0, b);
           }
         }
-        if (a.kc_app && lane == 0 && len + a.n_causal > a.Lmax)
-          record_error(a.err, SBD_DEVERR_CACHE_LEN);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&kv_full[stage]);
+        if (a.kc_app) {
+          // First iteration of a block: the causal rows' keys/values also
+          // enter the cache at len .. len + n_causal - 1 (positions >= len are
+          // read by no split of this call, or masked and zeroed where they
+          // are).  Plain copies, all of a batch's loads before its stores;
+          // nothing in this call waits for them.
+          if (len + a.n_causal <= a.Lmax) {
+            constexpr int kCpr = kSub * 8;             // 16-byte chunks per row
+            constexpr int kBatch = 8;                  // chunks per lane per batch
+            const int n_app = a.n_causal * kCpr;
+            for (int c0 = 0; c0 < n_app; c0 += 32 * kBatch) {
+              uint4 kv[kBatch], vv[kBatch];
+#pragma unroll
+              for (int e = 0; e < kBatch; ++e) {
+                const int c = c0 + e * 32 + lane;
+                if (c < n_app) {
+                  const size_t off = (((size_t)b * a.k + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
+                  kv[e] = *reinterpret_cast<const uint4*>(a.kb + off);
+                  vv[e] = *reinterpret_cast<const uint4*>(a.vb + off);
+                }
+              }
+#pragma unroll
+              for (int e = 0; e < kBatch; ++e) {
+                const int c = c0 + e * 32 + lane;
+                if (c < n_app) {
+                  const size_t dst =
+                      (((size_t)b * a.Lmax + len + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
+                  *reinterpret_cast<uint4*>(a.kc_app + dst) = kv[e];
+                  *reinterpret_cast<uint4*>(a.vc_app + dst) = vv[e];
+                }
+              }
+            }
+          } else if (lane == 0) {
+            record_error(a.err, SBD_DEVERR_CACHE_LEN);
+          }
+        }
       }
     }
   } else if (warp == 1) {
@@ -734,8 +741,24 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
                 : (R == 2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>);
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
+  // The block keys/values [B, k, Hkv, D] as 4-D tensors (D, Hkv, k, B), read
+  // in the cache tiles' boxes (64 columns x 64 rows, 128-byte swizzle): the
+  // rows past k are outside the tensor and arrive as zeros.
+  CUtensorMap kb_map, vb_map;
+  {
+    const uint64_t dims[4] = {(uint64_t)p.D, (uint64_t)p.Hkv, (uint64_t)p.k, (uint64_t)p.B};
+    const uint64_t strides[3] = {(uint64_t)p.D * 2, (uint64_t)p.Hkv * p.D * 2,
+                                 (uint64_t)p.k * p.Hkv * p.D * 2};
+    const uint32_t box[4] = {64, 1, (uint32_t)kTileKeys, 1};
+    sbd_status s = encode_tensor_map(&kb_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, (void*)kb, dims,
+                                     strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (s != SBD_OK) return s;
+    s = encode_tensor_map(&vb_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, (void*)vb, dims, strides,
+                          box, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (s != SBD_OK) return s;
+  }
   CUtensorMap k_map = tk, v_map = tv;
-  void* args[] = {(void*)&k_map, (void*)&v_map, (void*)&a};
+  void* args[] = {(void*)&k_map, (void*)&v_map, (void*)&kb_map, (void*)&vb_map, (void*)&a};
   return launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(kThreads), smem, st, args,
                     "attn_tc_kernel launch");
 }
