@@ -240,3 +240,22 @@ def test_kv_append_writes_only_the_new_rows():
     np.testing.assert_array_equal(lens, lens0)
     with pytest.raises(ValueError):
         oracle.kv_append(kc, vc, np.array([8, 0]), kr, vr)
+
+
+def test_empty_cache_and_one_block_key_return_its_value():
+    """A sequence with no cached keys and a block of one position: the only
+    key has softmax weight 1, so each query head returns its KV head's
+    block value exactly, whatever the query."""
+    q, kc, vc, lens, kb, vb = _rand_inputs(2, 1, 8, 2, 64, 5, seed=7, lens=[0, 0])
+    out = oracle.block_attention(q, kc, vc, lens, kb, vb)
+    for h in range(8):
+        np.testing.assert_allclose(out[:, 0, h], vb[:, 0, h // 4], rtol=0, atol=1e-15)
+
+
+def test_query_scale_trades_with_softmax_scale():
+    """s = scale * q.k: multiplying q by c and the scale by 1/c leaves every
+    score, hence the output, unchanged."""
+    q, kc, vc, lens, kb, vb = _rand_inputs(1, 4, 4, 2, 64, 40, seed=8, lens=[33])
+    a = oracle.block_attention(q, kc, vc, lens, kb, vb, scale=0.125)
+    b = oracle.block_attention(q * 4.0, kc, vc, lens, kb, vb, scale=0.125 / 4.0)
+    np.testing.assert_allclose(a, b, rtol=0, atol=1e-12)

@@ -111,3 +111,14 @@ def test_head_entropy_sample_rows_and_unmasked():
                 assert tok[b, i] == int(np.argmax(z + d["gumbel"][b, i].astype(np.float64)))
             else:
                 assert ent[b, i] == np.inf and tok[b, i] == -1
+
+
+def test_noise_dominates_at_large_tau():
+    """argmax(z + tau g): for tau far above the logit range the sampled token
+    is the argmax of the noise alone, which pins that tau scales the noise,
+    not the logits."""
+    rng = np.random.default_rng(3)
+    z = rng.standard_normal(50)
+    for t in range(20):
+        g = rng.gumbel(size=50)
+        assert oracle.sample_token(z, g, 1e9) == int(np.argmax(g))
