@@ -289,15 +289,20 @@ def lm_head_weight(w: Workload, seed: int) -> np.ndarray:
                             std=w.w_std), w.dtype)
 
 
-def hidden_states(w: Workload, seed: int, step: int = 0) -> np.ndarray:
-    """hidden [B,k,H]: rows N(0,1) times a per-row scale s drawn log-uniform
-    in [hidden_scale[0], hidden_scale[1]] (spreads the row entropies)."""
-    B, k, H = w.batch, w.block_k, w.hidden
-    h = normal_f32((B, k, H), seed, w.name, "hidden", step)
+def hidden_scales(w: Workload, seed: int, step: int = 0) -> np.ndarray:
+    """Per-row scale s [B,k] fp32, log-uniform in [hidden_scale[0],
+    hidden_scale[1]]: log s ~ U[log lo, log hi]."""
     g = _gen(seed, _key(w.name, "hidden_scale", step))
     lo, hi = np.log(w.hidden_scale[0]), np.log(w.hidden_scale[1])
-    s = np.exp(g.uniform(lo, hi, size=(B, k))).astype(np.float32)
-    h *= s[:, :, None]
+    return np.exp(g.uniform(lo, hi, size=(w.batch, w.block_k))).astype(np.float32)
+
+
+def hidden_states(w: Workload, seed: int, step: int = 0) -> np.ndarray:
+    """hidden [B,k,H]: rows N(0,1) times the per-row scale of hidden_scales
+    (spreads the row entropies), rounded to the storage type."""
+    B, k, H = w.batch, w.block_k, w.hidden
+    h = normal_f32((B, k, H), seed, w.name, "hidden", step)
+    h *= hidden_scales(w, seed, step)[:, :, None]
     return store(h, w.dtype)
 
 

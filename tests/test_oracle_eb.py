@@ -141,3 +141,58 @@ def test_steps_per_block_bounds():
             steps += 1
         assert 1 <= steps <= k
         assert (bt >= 0).all()
+
+
+# ------------------------------------------------------ margins to gamma
+
+def test_prefix_margins_worked_example():
+    """Sorted H = 0.01, 0.02, 0.5, 3.0 at gamma = 0.1: the decision on rank
+    j >= 2 compares S_{j-1} (the sum of the j-1 smallest) with gamma, so the
+    margins are |0.01 - 0.1|, |0.03 - 0.1|, |0.53 - 0.1| (by hand)."""
+    m = oracle.eb_prefix_margins([0.01, 0.02, 0.5, 3.0], 0.1)
+    assert np.allclose(m, [0.09, 0.07, 0.43], rtol=0, atol=1e-15)
+    # S_j and S_{j-1} differ: with S_j the first margin would be 0.07
+    m2 = oracle.eb_prefix_margins([0.2, 0.05], 0.1)
+    assert np.allclose(m2, [0.1], rtol=0, atol=1e-15)
+    assert oracle.eb_prefix_margins([0.7], 0.1) == []
+    assert oracle.eb_prefix_margins([], 0.1) == []
+
+
+def test_prefix_margins_equal_brute_force_thresholds():
+    """The margin of rank j is the distance from gamma to the smallest gamma
+    at which Eq. 9's bound admits j positions: min over subsets A with
+    |A| = j of (sum_A H - max_A H), found by enumeration."""
+    rng = np.random.default_rng(31)
+    for trial in range(60):
+        n = int(rng.integers(1, 8))
+        H = sorted(rng.exponential(0.2, n).tolist())
+        gamma = float(rng.choice(GAMMA_GRID))
+        m = oracle.eb_prefix_margins(H, gamma)
+        assert len(m) == max(0, n - 1)
+        for j in range(2, n + 1):
+            thr = min(sum(sorted(H[a] for a in A)[:-1])
+                      for A in itertools.combinations(range(n), j))
+            assert abs(m[j - 2] - abs(thr - gamma)) <= 1e-12, (H, gamma, j)
+
+
+def test_prefix_margins_locate_the_decision():
+    """Each margin is how far gamma may move before the accept count of
+    Eq. 3 changes at that rank: for rank j one of gamma +- margin is the
+    threshold c where eb_accept_count first admits j positions (admits j
+    just above c, fewer just below; "just" is 1e-12, far below the gaps
+    between prefix sums and above the rounding of gamma +- margin)."""
+    rng = np.random.default_rng(32)
+    for _ in range(80):
+        n = int(rng.integers(2, 10))
+        H = sorted(rng.exponential(0.15, n).tolist())
+        gamma = float(rng.uniform(0.0, 0.6))
+        m = oracle.eb_prefix_margins(H, gamma)
+        for j in range(2, n + 1):
+            hits = 0
+            for c in (gamma + m[j - 2], gamma - m[j - 2]):
+                if c < 0.0:
+                    continue
+                if (oracle.eb_accept_count(H, c + 1e-12) >= j
+                        and oracle.eb_accept_count(H, c - 1e-12) < j):
+                    hits += 1
+            assert hits >= 1, (H, gamma, j, m)

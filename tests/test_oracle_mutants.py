@@ -352,3 +352,39 @@ def _linear_corrected_shapes(block, batch, c=so.ROOFLINE_H100):
 def test_timing_model_mutants_are_caught(monkeypatch, name, mutant):
     _patch(monkeypatch, name, mutant)
     assert _fails(TR.test_every_printed_cell)
+
+
+# ------------------------------------------------------ EB margins to gamma
+
+def _margins_own_term(entropy_row_sorted, gamma):
+    out, prefix = [], 0.0
+    for j in range(1, len(entropy_row_sorted)):
+        prefix += float(entropy_row_sorted[j])      # S_j instead of S_{j-1}
+        out.append(abs(prefix - gamma))
+    return out
+
+
+def _margins_shifted(entropy_row_sorted, gamma):
+    out, prefix = [], 0.0
+    for j in range(len(entropy_row_sorted)):          # ranks start at 1, not 2
+        if j:
+            prefix += float(entropy_row_sorted[j - 1])
+        out.append(abs(prefix - gamma))
+    return out[:-1]
+
+
+def _margins_signed(entropy_row_sorted, gamma):
+    out, prefix = [], 0.0
+    for j in range(1, len(entropy_row_sorted)):
+        prefix += float(entropy_row_sorted[j - 1])
+        out.append(prefix - gamma)                   # no absolute value
+    return out
+
+
+@pytest.mark.parametrize("mutant", [_margins_own_term, _margins_shifted, _margins_signed])
+def test_margin_mutants_are_caught(monkeypatch, mutant):
+    _patch(monkeypatch, "eb_prefix_margins", mutant)
+    pins = [(TE.test_prefix_margins_worked_example, ()),
+            (TE.test_prefix_margins_equal_brute_force_thresholds, ()),
+            (TE.test_prefix_margins_locate_the_decision, ())]
+    assert all(_fails(fn, *args) for fn, args in pins[:2])
