@@ -608,21 +608,140 @@ def run_reference(args):
 
 # ------------------------------------------------------------------ sweep
 
+class SweepLoop:
+    """Device state and prepared ABI calls of the block-step loop of
+    Algorithm 3 over an n_layers-layer model: every block starts fully
+    masked; each step runs block attention over every layer's KV cache, the
+    LM head with entropy and Gumbel-max sampling over the still-masked
+    positions, and the EB select; steps repeat until no position of any
+    sequence is masked (one 4-byte read of the remaining count per step).
+
+    The per-layer caches and the other large inputs are drawn on the device
+    with PyTorch's seeded generator.  Hidden rows are drawn per step of a
+    block (hidden[s] feeds step s); the Gumbel noise of a block is drawn
+    once and indexed by block position, so each committed token is a
+    Gumbel-max sample at its commit step.  With noise="philox" the LM-head
+    kernel generates the noise itself, with counter offset s at step s."""
+
+    def __init__(self, w: "gen.Workload", seed: int, noise: str, tau: float, gamma: float,
+                 dev, stream):
+        import ctypes
+
+        import torch
+
+        import paper_2509_04185_gb300 as sbd
+        self.sbd, self.w, self.stream = sbd, w, stream
+        self.noise, self.tau, self.gamma, self.seed = noise, tau, gamma, seed
+        B, k, Hq, Hkv, D, L = (w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim,
+                               w.max_cache_len)
+        V, H, NL = w.vocab, w.hidden, w.n_layers
+        g = torch.Generator(device=dev)
+        g.manual_seed(seed * 1000003 + 17)
+
+        def randn(*shape, std=1.0):
+            return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32)
+                    * std).bfloat16()
+
+        self.layers = []
+        for _ in range(NL):
+            self.layers.append(dict(q=randn(B, k, Hq, D), kc=randn(B, L, Hkv, D),
+                                    vc=randn(B, L, Hkv, D), kb=randn(B, k, Hkv, D),
+                                    vb=randn(B, k, Hkv, D)))
+        self.lens = torch.full((B,), L, dtype=torch.int32, device=dev)
+        self.W = randn(V, H, std=w.w_std)
+        lo, hi = np.log(w.hidden_scale[0]), np.log(w.hidden_scale[1])
+        self.hidden = []
+        for _ in range(k):
+            h = torch.randn(B, k, H, generator=g, device=dev)
+            sc = torch.exp(torch.empty(B, k, 1, device=dev).uniform_(lo, hi, generator=g))
+            self.hidden.append((h * sc).bfloat16())
+        u = torch.rand(B, k, V, generator=g, device=dev, dtype=torch.float64).clamp_(
+            1e-300, 1 - 1e-16)
+        self.gumbel = (-torch.log(-torch.log(u))).float()
+        del u
+        self.outs = [torch.empty_like(self.layers[0]["q"]) for _ in range(NL)]
+        self.masked = torch.ones(B, k, dtype=torch.uint8, device=dev)
+        self.bt = torch.full((B, k), -1, dtype=torch.int32, device=dev)
+        self.ent = torch.empty(B, k, dtype=torch.float32, device=dev)
+        self.tok = torch.empty(B, k, dtype=torch.int32, device=dev)
+        self.n_un = torch.empty(B, dtype=torch.int32, device=dev)
+        self.left_h = torch.empty(1, dtype=torch.int32).pin_memory()
+        ad = sbd.attn_desc(self.layers[0]["q"], self.layers[0]["kc"])
+        self.ws_a = torch.empty(max(1, sbd.lib.sbd_block_attention_workspace_size(
+            ctypes.byref(ad))), dtype=torch.uint8, device=dev)
+        hd = sbd.head_desc(self.hidden[0], self.W)
+        self.ws_h = torch.empty(max(1, sbd.lib.sbd_head_entropy_sample_workspace_size(
+            ctypes.byref(hd))), dtype=torch.uint8, device=dev)
+        self.attn_calls = [
+            sbd.prepare_block_attention(L_["q"], L_["kc"], L_["vc"], self.lens, L_["kb"],
+                                        L_["vb"], self.outs[i], self.ws_a, stream=stream)
+            for i, L_ in enumerate(self.layers)]
+        if noise == "philox":
+            self.head_calls = [
+                sbd.prepare_head_entropy_sample_philox(self.hidden[s_], self.W, self.masked, seed,
+                                                       s_, tau, self.ent, self.tok, self.ws_h,
+                                                       stream=stream)
+                for s_ in range(k)]
+        else:
+            self.head_calls = [
+                sbd.prepare_head_entropy_sample(self.hidden[s_], self.W, self.masked, self.gumbel,
+                                                tau, self.ent, self.tok, self.ws_h, stream=stream)
+                for s_ in range(k)]
+        self.eb_call = sbd.prepare_eb_select(self.ent, self.tok, gamma, self.masked, self.bt,
+                                             self.n_un, stream=stream)
+
+    def launches_per_step(self) -> int:
+        """Kernels one step launches: per layer the attention kernel (+ the
+        split combine when the workspace is in use), the head's compaction,
+        main and combine kernels, and the EB select."""
+        return self.w.n_layers * (2 if self.ws_a.numel() > 1 else 1) + 3 + 1
+
+    def block(self, ev=None, trace=None) -> int:
+        """One block: steps until no masks.  Returns the step count.  ev:
+        a list that gets four CUDA events per step (start, after attention,
+        after the head, after EB).  trace: a list that gets, per step, host
+        copies of the block state before and after the step and of the
+        head's outputs (this adds synchronisation; tests only)."""
+        import torch
+        k = self.w.block_k
+        stream = self.stream
+        self.masked.fill_(1)
+        self.bt.fill_(-1)
+        steps = 0
+        while True:
+            if trace is not None:
+                stream.synchronize()
+                before = (self.masked.cpu().numpy(), self.bt.cpu().numpy())
+            if ev is not None:
+                ev.append([torch.cuda.Event(enable_timing=True) for _ in range(4)])
+                ev[-1][0].record(stream)
+            for c in self.attn_calls:
+                c()
+            if ev is not None:
+                ev[-1][1].record(stream)
+            self.head_calls[min(steps, k - 1)]()
+            if ev is not None:
+                ev[-1][2].record(stream)
+            self.eb_call()
+            if ev is not None:
+                ev[-1][3].record(stream)
+            self.left_h.copy_(self.masked.sum(dtype=torch.int32).view(1), non_blocking=True)
+            stream.synchronize()
+            if trace is not None:
+                trace.append(dict(step=steps, masked_before=before[0], bt_before=before[1],
+                                  entropy=self.ent.cpu().numpy(), token=self.tok.cpu().numpy(),
+                                  masked_after=self.masked.cpu().numpy(),
+                                  bt_after=self.bt.cpu().numpy(),
+                                  n_unmasked=self.n_un.cpu().numpy()))
+            steps += 1
+            if int(self.left_h.item()) == 0 or steps >= k:
+                return steps
+
+
 def run_sweep(args):
     """The 32-layer block-step loop at Llama-3.1-8B attention shapes
-    (Algorithm 3): every block starts fully masked; each step runs block
-    attention over all 32 layers' KV caches, the LM head with entropy and
-    Gumbel-max sampling over the still-masked positions, and the EB select;
-    steps repeat until no position of any sequence is masked (one 4-byte
-    read of the remaining count per step).  A timed step is one such
-    iteration; the timed region covers whole blocks.
-
-    The 17 GB of per-layer caches and the other large inputs are drawn on the
-    device with PyTorch's seeded generator (the parity tests use the host
-    generator on one layer of the same shapes).  Hidden rows are redrawn per
-    step; the Gumbel noise of a block is drawn once and indexed by block
-    position, so each committed token is a Gumbel-max sample at its commit
-    step."""
+    (Algorithm 3), driven by SweepLoop.  A timed step is one iteration of
+    the loop; the timed region covers whole blocks."""
     import torch
 
     import paper_2509_04185_gb300 as sbd
@@ -636,79 +755,9 @@ def run_sweep(args):
     w = gen.get_workload(args.workload)
     B, k, Hq, Hkv, D, L = w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim, w.max_cache_len
     V, H, NL = w.vocab, w.hidden, w.n_layers
-    g = torch.Generator(device=dev)
-    g.manual_seed(args.seed * 1000003 + 17)
-
-    def randn(*shape, std=1.0):
-        return (torch.randn(*shape, generator=g, device=dev, dtype=torch.float32) * std).bfloat16()
-
-    layers = []
-    for _ in range(NL):
-        layers.append(dict(q=randn(B, k, Hq, D), kc=randn(B, L, Hkv, D), vc=randn(B, L, Hkv, D),
-                           kb=randn(B, k, Hkv, D), vb=randn(B, k, Hkv, D)))
-    lens = torch.full((B,), L, dtype=torch.int32, device=dev)
-    Wt = randn(V, H, std=w.w_std)
-    lo, hi = np.log(w.hidden_scale[0]), np.log(w.hidden_scale[1])
-    hidden = []
-    for _ in range(k):
-        h = torch.randn(B, k, H, generator=g, device=dev)
-        sc = torch.exp(torch.empty(B, k, 1, device=dev).uniform_(lo, hi, generator=g))
-        hidden.append((h * sc).bfloat16())
-    u = torch.rand(B, k, V, generator=g, device=dev, dtype=torch.float64).clamp_(1e-300, 1 - 1e-16)
-    gumbel = (-torch.log(-torch.log(u))).float()
-    del u
-    outs = [torch.empty_like(layers[0]["q"]) for _ in range(NL)]
-    masked = torch.ones(B, k, dtype=torch.uint8, device=dev)
-    bt = torch.full((B, k), -1, dtype=torch.int32, device=dev)
-    ent = torch.empty(B, k, dtype=torch.float32, device=dev)
-    tok = torch.empty(B, k, dtype=torch.int32, device=dev)
-    n_un = torch.empty(B, dtype=torch.int32, device=dev)
-    left_h = torch.empty(1, dtype=torch.int32).pin_memory()
     stream = torch.cuda.current_stream(dev)
-    import ctypes
-    ad = sbd.attn_desc(layers[0]["q"], layers[0]["kc"])
-    ws_a = torch.empty(max(1, sbd.lib.sbd_block_attention_workspace_size(ctypes.byref(ad))),
-                       dtype=torch.uint8, device=dev)
-    hd = sbd.head_desc(hidden[0], Wt)
-    ws_h = torch.empty(max(1, sbd.lib.sbd_head_entropy_sample_workspace_size(ctypes.byref(hd))),
-                       dtype=torch.uint8, device=dev)
-    attn_calls = [sbd.prepare_block_attention(L_["q"], L_["kc"], L_["vc"], lens, L_["kb"], L_["vb"],
-                                              outs[i], ws_a, stream=stream)
-                  for i, L_ in enumerate(layers)]
-    if args.noise == "philox":
-        # in-kernel noise: a fresh counter offset per step of the block
-        head_calls = [sbd.prepare_head_entropy_sample_philox(hidden[s_], Wt, masked, args.seed, s_,
-                                                             args.tau, ent, tok, ws_h, stream=stream)
-                      for s_ in range(k)]
-    else:
-        head_calls = [sbd.prepare_head_entropy_sample(hidden[s_], Wt, masked, gumbel, args.tau, ent,
-                                                      tok, ws_h, stream=stream) for s_ in range(k)]
-    eb_call = sbd.prepare_eb_select(ent, tok, args.gamma, masked, bt, n_un, stream=stream)
-
-    def block(ev=None):
-        """One block: steps until no masks.  Returns the step count."""
-        masked.fill_(1)
-        bt.fill_(-1)
-        steps = 0
-        while True:
-            if ev is not None:
-                ev.append([torch.cuda.Event(enable_timing=True) for _ in range(4)])
-                ev[-1][0].record(stream)
-            for c in attn_calls:
-                c()
-            if ev is not None:
-                ev[-1][1].record(stream)
-            head_calls[min(steps, k - 1)]()
-            if ev is not None:
-                ev[-1][2].record(stream)
-            eb_call()
-            if ev is not None:
-                ev[-1][3].record(stream)
-            left_h.copy_(masked.sum(dtype=torch.int32).view(1), non_blocking=True)
-            stream.synchronize()
-            steps += 1
-            if int(left_h.item()) == 0 or steps >= k:
-                return steps
+    loop = SweepLoop(w, args.seed, args.noise, args.tau, args.gamma, dev, stream)
+    block = loop.block
 
     sampler = ClockSampler(local_rank) if rank == 0 else None
     if sampler:
@@ -767,7 +816,7 @@ def run_sweep(args):
         "steps_per_block": round(n_steps / n_blocks, 3),
         "blocks": n_blocks,
         "tokens_committed_per_s": round(n_blocks * B * k / (total_ms * 1e-3) * world, 1),
-        "gpu_launches": int(n_steps * (NL * (2 if ws_a.numel() > 1 else 1) + 3 + 1)),
+        "gpu_launches": int(n_steps * loop.launches_per_step()),
         "per_call_us": {"attention_32_layers": round(attn_ms * 1000, 3),
                         "head": round(head_ms * 1000, 3), "eb_select": round(eb_ms * 1000, 3)},
         "roofline": {

@@ -38,27 +38,14 @@ using namespace sbd_dev;
 
 constexpr int kTileKeys = 64;
 constexpr int kMaxStages = 4;
-// Ring depth cap and the key-group count used for 4 row tiles (64 packed
-// rows); defaults chosen by measurement.
-#ifndef SBD_ATTN_STAGE_CAP
-#define SBD_ATTN_STAGE_CAP 3
-#endif
-#ifndef SBD_ATTN_KG_MT4
-#define SBD_ATTN_KG_MT4 1
-#endif
-// bf16 attention on the tcgen05 kernel (block_attention_tc.cu) rather than
-// the mma.sync kernel of this file, from this many packed rows on.
-#ifndef SBD_ATTN_TC
-#define SBD_ATTN_TC 1
-#endif
+// Ring depth cap (chosen by measurement).
+constexpr int kStageCap = 3;
 // Largest batch for which the CTAs of a multi-wave launch take the
-// sequences longest first (0: never).
-#ifndef SBD_ATTN_ORDER_MAX_B
-#define SBD_ATTN_ORDER_MAX_B 128
-#endif
-#ifndef SBD_ATTN_TC_MIN_ROWS
-#define SBD_ATTN_TC_MIN_ROWS 17
-#endif
+// sequences longest first.
+constexpr int kOrderMaxB = 128;
+// bf16 attention runs on the tcgen05 kernel (block_attention_tc.cu) rather
+// than the mma.sync kernel of this file from this many packed rows on.
+constexpr int kTcMinRows = 17;
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------ mma helpers
@@ -665,16 +652,16 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
   }
   // With more CTAs than one wave, the CTAs take the sequences longest first
   // (the pick costs B^2 comparisons per CTA, hence the batch limit).
-  p.order = p.bf16 && p.B > 1 && p.B <= SBD_ATTN_ORDER_MAX_B &&
+  p.order = p.bf16 && p.B > 1 && p.B <= kOrderMaxB &&
             (long long)p.B * p.Hkv * p.splits > num_sms();
   // Ring depth: as many stages as a split has tiles, between 2 and 4.
   const int per_split = (tiles + p.splits - 1) / p.splits;
-  const int cap = SBD_ATTN_STAGE_CAP < kMaxStages ? SBD_ATTN_STAGE_CAP : kMaxStages;
+  const int cap = kStageCap < kMaxStages ? kStageCap : kMaxStages;
   p.stages = per_split < 2 ? 2 : (per_split > cap ? cap : per_split);
   // Row tiles of 16 packed rows; small tiles also split every key tile
   // between key groups so that at least 4 (up to 8) warps share the work.
   p.MT = (p.M + 15) / 16;
-  p.KG = p.MT >= 5 ? 1 : (p.MT == 4 ? SBD_ATTN_KG_MT4 : (p.MT == 3 ? 2 : 4));
+  p.KG = p.MT >= 5 ? 1 : (p.MT == 4 ? 1 : (p.MT == 3 ? 2 : 4));
   if (p.MT == 1) p.KG = 4;
   return p;
 }
@@ -758,7 +745,7 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   // copied into 4, 2 or 1 TMEM lane quadrants so that all SM sub-partitions
   // share the softmax.  Batch 16, KV 8192: 32 rows (k = 8) 115 -> 110 us;
   // 16 rows (k = 4) 104 us on mma.sync against 108 us on tcgen05.
-  if (SBD_ATTN_TC && p.M >= SBD_ATTN_TC_MIN_ROWS) {
+  if (p.M >= kTcMinRows) {
     s = attn_tc_launch(p, tk, tv, q, lens, kb, vb, out, a.part_o, a.part_lse, kc_app, vc_app,
                        st);
     if (s != SBD_OK) return s;

@@ -51,13 +51,6 @@ constexpr int kRows = 128;                 // MMA M (packed rows, padded)
 constexpr int kSoftWarps = 8;              // two per TMEM lane quadrant
 constexpr int kThreads = 64 + 32 * kSoftWarps;   // producer, MMA, softmax warps
 constexpr float kRescaleThreshold = 8.f;   // log2 units
-// Cache tiles can be prefetched into L2 this many tiles ahead of the ring.
-// Off by default: with one wave of long CTAs the extra requests measured
-// slower (batch 16 x 8192 cache, k = 16: 128 us per layer without, 152 us
-// with 8 tiles ahead).
-#ifndef SBD_ATTN_L2_AHEAD
-#define SBD_ATTN_L2_AHEAD 0
-#endif
 
 // ------------------------------------------------------------ tcgen05 PTX
 __device__ __forceinline__ void tc_alloc(uint32_t* dst_smem, uint32_t ncols) {
@@ -289,16 +282,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         tma_prefetch_desc(&tmap_vb);
       }
     }
-    auto prefetch = [&](int t) {
-      if (SBD_ATTN_L2_AHEAD > 0 && t < t_end && t < n_cache_tiles) {
-        for (int h = 0; h < kSub; ++h) {
-          tma_prefetch_l2_4d(&tmap_k, 64 * h, hkv, t * kTileKeys, b);
-          tma_prefetch_l2_4d(&tmap_v, 64 * h, hkv, t * kTileKeys, b);
-        }
-      }
-    };
-    if (lane == 0)
-      for (int t = t_begin + kStages; t < t_begin + kStages + SBD_ATTN_L2_AHEAD; ++t) prefetch(t);
     for (int j = 0; j < n; ++j) {
       const int t = t_begin + j;
       const int stage = j % kStages;
@@ -313,7 +296,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         const bool tail = valid < kTileKeys;
         uint64_t* bar = tail ? &tail_bar : &kv_full[stage];
         if (lane == 0) {
-          prefetch(t + kStages + SBD_ATTN_L2_AHEAD);
           mbar_arrive_expect_tx(bar, 2 * kSub * kKVSub);
           for (int h = 0; h < kSub; ++h) {
             tma_load_4d(smem_raw + (k_chunk(j, h) - smem_u32(smem_raw)), &tmap_k, bar, 64 * h, hkv,

@@ -20,23 +20,32 @@ static __device__ __align__(256) unsigned char g_head_scratch[SBD_HEAD_NOALLOC_M
 
 constexpr int kMaxDevices = 64;
 
+// The device address of the array, per device, kept once it was obtained; a
+// failed lookup is not kept, so the next call tries again.
 struct ScratchTable {
-  std::once_flag once[kMaxDevices];
+  std::mutex mu;
   void* ptr[kMaxDevices] = {nullptr};
-  cudaError_t err[kMaxDevices] = {cudaSuccess};
 };
 ScratchTable& table() {
   static ScratchTable t;
   return t;
 }
 
-// Once per device, with that device current: the device address of the array.
-void resolve(int dev) {
-  void* p = nullptr;
-  cudaError_t e = cudaGetSymbolAddress(&p, g_head_scratch);
-  table().err[dev] = e;
-  table().ptr[dev] = e == cudaSuccess ? p : nullptr;
-  if (e != cudaSuccess) cudaGetLastError();
+// With device `dev` current: its address of the array, looked up on first use.
+sbd_status scratch_address(int dev, void** out) {
+  ScratchTable& t = table();
+  std::lock_guard<std::mutex> lock(t.mu);
+  if (!t.ptr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_head_scratch);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return sbd::cuda_fail(e, "cudaGetSymbolAddress(no-allocation scratch)");
+    }
+    t.ptr[dev] = p;
+  }
+  *out = t.ptr[dev];
+  return SBD_OK;
 }
 
 }  // namespace
@@ -47,7 +56,13 @@ extern "C" sbd_status sbd_head_entropy_sample_noalloc(const sbd_head_desc* desc,
                                                       float tau, float* entropy, int32_t* token,
                                                       void* stream) {
   // An invalid descriptor reports 0 here and is diagnosed by the call below.
-  const size_t need = sbd_head_entropy_sample_workspace_size(desc);
+  // The floor needs no device, so a shape too large for any device is
+  // rejected even before the device is queried.
+  size_t need = desc ? sbd::head_workspace_floor(*desc) : 0;
+  if (need <= (size_t)SBD_HEAD_NOALLOC_MAX_SCRATCH) {
+    const size_t exact = sbd_head_entropy_sample_workspace_size(desc);
+    if (exact > need) need = exact;
+  }
   if (need > (size_t)SBD_HEAD_NOALLOC_MAX_SCRATCH)
     return sbd::fail(SBD_ERR_UNSUPPORTED,
                      "this shape needs %zu bytes of scratch; the no-allocation variant holds "
@@ -58,9 +73,9 @@ extern "C" sbd_status sbd_head_entropy_sample_noalloc(const sbd_head_desc* desc,
   if (e != cudaSuccess) return sbd::cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices)
     return sbd::fail(SBD_ERR_UNSUPPORTED, "device ordinal %d >= %d", dev, kMaxDevices);
-  std::call_once(table().once[dev], resolve, dev);
-  if (!table().ptr[dev])
-    return sbd::cuda_fail(table().err[dev], "cudaGetSymbolAddress(no-allocation scratch)");
-  return sbd_head_entropy_sample(desc, hidden, w, masked, gumbel, tau, entropy, token,
-                                 table().ptr[dev], (size_t)SBD_HEAD_NOALLOC_MAX_SCRATCH, stream);
+  void* scratch = nullptr;
+  const sbd_status st = scratch_address(dev, &scratch);
+  if (st != SBD_OK) return st;
+  return sbd_head_entropy_sample(desc, hidden, w, masked, gumbel, tau, entropy, token, scratch,
+                                 (size_t)SBD_HEAD_NOALLOC_MAX_SCRATCH, stream);
 }

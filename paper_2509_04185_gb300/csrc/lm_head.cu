@@ -42,39 +42,17 @@ constexpr int kABytes = kBM * kBK * 2;  // one W box
 constexpr int kMaxStages = 16;
 // A pipeline stage holds up to this many consecutive boxes along the hidden
 // dimension (longer contiguous reads of every W row per stage), and the ring
-// gets this many bytes of shared memory.
-// Hidden rows are loaded in boxes of up to 128 rows (1), or of 16 only (0).
-#ifndef SBD_HEAD_BIG_BOXES
-#define SBD_HEAD_BIG_BOXES 1
-#endif
-#ifndef SBD_HEAD_MAX_BOXES
-#define SBD_HEAD_MAX_BOXES 4
-#endif
-#ifndef SBD_HEAD_RING_BYTES
-#define SBD_HEAD_RING_BYTES (216 * 1024)
-#endif
-// Resident CTAs per SM (the ring budget is shared between them) and whether
-// W is loaded with an L2 evict-first policy.
-#ifndef SBD_HEAD_CTAS_PER_SM
-#define SBD_HEAD_CTAS_PER_SM 1
-#endif
-#ifndef SBD_HEAD_EVICT_FIRST
-#define SBD_HEAD_EVICT_FIRST 1
-#endif
-// Epilogue warps: 4 or 8 (warps 2, 3, ...; warp w reads TMEM lanes of
-// quadrant w % 4, and the warps of one quadrant take alternate 16-column
-// chunks).
-#ifndef SBD_HEAD_EPI_WARPS
-#define SBD_HEAD_EPI_WARPS 8
-#endif
-constexpr int kEpiWarps = SBD_HEAD_EPI_WARPS;
+// gets this many bytes of shared memory.  One CTA per SM; W is loaded with
+// an L2 evict-first policy, the hidden rows (re-read by every CTA) in boxes
+// of up to 128 rows.
+constexpr int kMaxBoxes = 4;
+constexpr int kRingBytes = 216 * 1024;
+// Epilogue warps (warps 2, 3, ...): warp w reads the TMEM lanes of quadrant
+// w % 4, and the two warps of one quadrant take alternate 16-column chunks.
+constexpr int kEpiWarps = 8;
 // Chunks of Gumbel noise an epilogue warp keeps in flight ahead of the one
 // it reduces (loads from HBM take longer than the reduction of one chunk).
-#ifndef SBD_HEAD_G_AHEAD
-#define SBD_HEAD_G_AHEAD 2
-#endif
-constexpr int kGAhead = SBD_HEAD_G_AHEAD;
-static_assert(kEpiWarps == 4 || kEpiWarps == 8, "4 or 8 epilogue warps");
+constexpr int kGAhead = 2;
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kHeadThreads = 64 + kEpiThreads;   // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr float kLog2e = 1.4426950408889634f;
@@ -351,7 +329,7 @@ struct HeadArgs {
 // y = x W^T in bf16 (all rows of x live, no compaction, no noise); the
 // epilogue stores the accumulators instead of reducing them.
 template <bool kPhilox, bool kLinear>
-__global__ void __launch_bounds__(kHeadThreads, SBD_HEAD_CTAS_PER_SM)
+__global__ void __launch_bounds__(kHeadThreads, 1)
 head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                const __grid_constant__ CUtensorMap tmap_h,
                const __grid_constant__ CUtensorMap tmap_h64,
@@ -406,7 +384,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int ksplit = kLinear ? a.ksplit : 1;
   const int n_units = a.n_tiles * ksplit;
   auto fits = [&](int bx, int n_st) { return ring_bytes / (bx * (kABytes + b_box)) >= n_st; };
-  int boxes = SBD_HEAD_MAX_BOXES;
+  int boxes = kMaxBoxes;
   while (boxes > 1 &&
          ((a.H / kBK) % (boxes * ksplit) != 0 || !fits(boxes, boxes > 2 ? 3 : 2)))
     boxes >>= 1;
@@ -461,12 +439,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
             mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
             for (int x = 0; x < boxes; ++x) {
               const int col = ((kb0 + kb) * boxes + x) * kBK;
-#if SBD_HEAD_EVICT_FIRST
               tma_load_2d_hint(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM, policy);
-#else
-              (void)policy;
-              tma_load_2d(st + x * kABytes, &tmap_w, &full_bar[s], col, tile * kBM);
-#endif
               // the n_eff hidden rows the MMA reads, in the tallest boxes that
               // fit: these rows come from L2 for every vocabulary tile, where
               // the copy rate per SM grows with the box size
@@ -818,11 +791,11 @@ HeadWs head_ws_layout(const sbd::HeadPlan& p, void* base) {
 }
 
 
-// Shared memory of the ring: SBD_HEAD_RING_BYTES per SM, within what a CTA
-// can have next to the epilogue scratch.
+// Shared memory of the ring: kRingBytes, within what a CTA can have next to
+// the epilogue scratch.
 int head_ring_bytes(int rows_alloc) {
-  const int per_cta = (224 * 1024) / SBD_HEAD_CTAS_PER_SM - 1024 - 1024;
-  int budget = SBD_HEAD_RING_BYTES / SBD_HEAD_CTAS_PER_SM;
+  const int per_cta = 224 * 1024 - 1024 - 1024;
+  int budget = kRingBytes;
   if (budget > per_cta - head_scratch_bytes(rows_alloc)) budget = per_cta - head_scratch_bytes(rows_alloc);
   return budget;
 }
@@ -859,7 +832,7 @@ HeadPlan head_plan(const sbd_head_desc& d) {
   p.rows_alloc = bk <= 16 ? 16 : ((bk + 15) / 16) * 16;
   const int n_tiles = (d.vocab + kBM - 1) / kBM;
   if (p.bf16) {
-    const int slots = num_sms() * SBD_HEAD_CTAS_PER_SM;
+    const int slots = num_sms();
     p.n_ctas = n_tiles < slots ? n_tiles : slots;
   } else {
     p.n_ctas = n_tiles;
@@ -868,6 +841,23 @@ HeadPlan head_plan(const sbd_head_desc& d) {
 }
 
 size_t head_workspace_bytes(const HeadPlan& p) { return head_ws_layout(p, nullptr).bytes; }
+
+size_t head_workspace_floor(const sbd_head_desc& d) {
+  if (d.batch < 0 || d.block_k < 1 || d.hidden < 1 || d.vocab < 1 ||
+      (long long)d.batch * d.block_k > 512 ||
+      (d.dtype != SBD_DTYPE_F32 && d.dtype != SBD_DTYPE_BF16))
+    return 0;
+  HeadPlan p;
+  p.B = d.batch;
+  p.k = d.block_k;
+  p.H = d.hidden;
+  p.V = d.vocab;
+  p.bf16 = d.dtype == SBD_DTYPE_BF16;
+  const int bk = d.batch * d.block_k;
+  p.rows_alloc = bk <= 16 ? 16 : ((bk + 15) / 16) * 16;
+  p.n_ctas = 1;
+  return head_ws_layout(p, nullptr).bytes;
+}
 
 sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
                        const uint8_t* masked, const float* gumbel, float tau, float* entropy,
@@ -944,7 +934,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.linear_rows = 0;
     a.ksplit = 1;
     a.part_y = nullptr;
-    a.h_big = SBD_HEAD_BIG_BOXES ? (p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16)) : 16;
+    a.h_big = p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16);
     a.ring_bytes = head_ring_bytes(p.rows_alloc);
     // tensor memory for two accumulators of the allocated width (one of it
     // above 256 rows); the kernel picks the buffer count from the live rows
@@ -1021,7 +1011,7 @@ int linear_ksplit(int T, int K, int N) {
   // T x 128 fp32 partials, and the sum over ranges reads them all back in
   // a second launch.  The split with the shortest modelled time wins.
   const int max_ks = linear_max_split(T, K, N);
-  const int sms = num_sms() * SBD_HEAD_CTAS_PER_SM;
+  const int sms = num_sms();
   const int n_tiles = (N + kBM - 1) / kBM;
   const double n_eff = T <= 16 ? 16.0 : (double)((T + 15) / 16 * 16);
   const double t_mem = 128.0 * K * 2 / 45e3, t_mma = 2.0 * 128 * n_eff * K / 14.8e6;  // us
@@ -1089,7 +1079,7 @@ sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void
   a.H = K;
   a.rows_alloc = rows_alloc;
   a.n_tiles = (N + kBM - 1) / kBM;
-  a.h_big = SBD_HEAD_BIG_BOXES ? (T >= 128 ? 128 : (T >= 64 ? 64 : 16)) : 16;
+  a.h_big = T >= 128 ? 128 : (T >= 64 ? 64 : 16);
   a.ring_bytes = head_ring_bytes(rows_alloc);
   const int n_acc_alloc = 2 * rows_alloc <= 512 ? 2 : 1;
   uint32_t cols = 32;
@@ -1104,7 +1094,7 @@ sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void
   const void* fn = (const void*)head_tc_kernel<false, true>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel, linear)");
-  const int slots = num_sms() * SBD_HEAD_CTAS_PER_SM;
+  const int slots = num_sms();
   const int units = a.n_tiles * ksplit;
   const int n_ctas = units < slots ? units : slots;
   void* args[] = {(void*)&tw, (void*)&tx, (void*)&tx64, (void*)&tx128, (void*)&a};

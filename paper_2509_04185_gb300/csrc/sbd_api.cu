@@ -16,8 +16,12 @@ thread_local char g_last_error[512] = "";
 constexpr int kMaxDevices = 64;
 __device__ int g_device_error = 0;
 
+// Per device: the SM count and the device address of the error word, set
+// once both queries have succeeded (a failed query is retried on the next
+// call instead of being kept).
 struct DeviceCache {
-  std::once_flag once[kMaxDevices];
+  std::mutex mu;
+  bool ready[kMaxDevices] = {false};
   int sms[kMaxDevices] = {0};
   int* err_word[kMaxDevices] = {nullptr};
 };
@@ -29,26 +33,45 @@ DeviceCache& cache() {
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 
-void init_device(int dev) {
-  int sms = 0;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) sms = 0;
-  cache().sms[dev] = sms;
-  void* p = nullptr;
-  if (cudaGetSymbolAddress(&p, g_device_error) == cudaSuccess)
-    cache().err_word[dev] = static_cast<int*>(p);
-  else
-    cudaGetLastError();
-}
-
-int current_device() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  return dev < kMaxDevices ? dev : 0;
+// The current device's ordinal; an error status (with the reason recorded)
+// when it cannot be read or is beyond the table.
+sbd_status current_device(int* dev) {
+  cudaError_t e = cudaGetDevice(dev);
+  if (e != cudaSuccess) return sbd::cuda_fail(e, "cudaGetDevice");
+  if (*dev < 0 || *dev >= kMaxDevices)
+    return sbd::fail(SBD_ERR_UNSUPPORTED, "device ordinal %d >= %d", *dev, kMaxDevices);
+  return SBD_OK;
 }
 
 }  // namespace
 
 namespace sbd {
+
+sbd_status device_ready() {
+  int dev = 0;
+  const sbd_status st = current_device(&dev);
+  if (st != SBD_OK) return st;
+  DeviceCache& c = cache();
+  std::lock_guard<std::mutex> lock(c.mu);
+  if (c.ready[dev]) return SBD_OK;
+  int sms = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess || sms <= 0) {
+    cudaGetLastError();
+    return e != cudaSuccess ? cuda_fail(e, "cudaDeviceGetAttribute(MultiProcessorCount)")
+                            : fail(SBD_ERR_CUDA, "device %d reports %d SMs", dev, sms);
+  }
+  void* p = nullptr;
+  e = cudaGetSymbolAddress(&p, g_device_error);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return cuda_fail(e, "cudaGetSymbolAddress(device error word)");
+  }
+  c.sms[dev] = sms;
+  c.err_word[dev] = static_cast<int*>(p);
+  c.ready[dev] = true;
+  return SBD_OK;
+}
 
 sbd_status fail(sbd_status st, const char* fmt, ...) {
   va_list ap;
@@ -62,16 +85,20 @@ sbd_status cuda_fail(cudaError_t e, const char* what) {
   return fail(SBD_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
 }
 
+// Both below are called only after device_ready() succeeded on this thread's
+// current device (every launching entry point checks it first).
 int num_sms() {
-  const int dev = current_device();
-  std::call_once(cache().once[dev], init_device, dev);
-  return cache().sms[dev] > 0 ? cache().sms[dev] : 1;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
+  std::lock_guard<std::mutex> lock(cache().mu);
+  return cache().ready[dev] ? cache().sms[dev] : 1;
 }
 
 int* device_error_word() {
-  const int dev = current_device();
-  std::call_once(cache().once[dev], init_device, dev);
-  return cache().err_word[dev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(cache().mu);
+  return cache().ready[dev] ? cache().err_word[dev] : nullptr;
 }
 
 sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32_t rank,
@@ -189,6 +216,8 @@ sbd_status attn_call(const sbd_attn_desc* desc, int n_causal, const void* q, con
     if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
     if (!aligned16(ptrs[i])) return fail(SBD_ERR_INVALID_ARG, "%s is not 16-byte aligned", names[i]);
   }
+  s = sbd::device_ready();
+  if (s != SBD_OK) return s;
   sbd::AttnPlan p = sbd::attn_plan(*desc);
   p.n_causal = n_causal;
   const size_t need = sbd::attn_workspace_bytes(p);
@@ -207,7 +236,7 @@ sbd_status attn_call(const sbd_attn_desc* desc, int n_causal, const void* q, con
 extern "C" {
 
 size_t sbd_block_attention_workspace_size(const sbd_attn_desc* desc) {
-  if (check_attn_desc(desc) != SBD_OK) return 0;
+  if (check_attn_desc(desc) != SBD_OK || sbd::device_ready() != SBD_OK) return 0;
   return sbd::attn_workspace_bytes(sbd::attn_plan(*desc));
 }
 
@@ -233,7 +262,7 @@ sbd_status sbd_block_attention_causal_prefix(const sbd_attn_desc* desc, int32_t 
 }
 
 size_t sbd_head_entropy_sample_workspace_size(const sbd_head_desc* desc) {
-  if (check_head_desc(desc) != SBD_OK) return 0;
+  if (check_head_desc(desc) != SBD_OK || sbd::device_ready() != SBD_OK) return 0;
   return sbd::head_workspace_bytes(sbd::head_plan(*desc));
 }
 
@@ -262,6 +291,8 @@ sbd_status head_call(const sbd_head_desc* desc, const void* hidden, const void* 
     return fail(SBD_ERR_INVALID_ARG, "gumbel is NULL but tau != 0");
   if (gumbel && !aligned16(gumbel))
     return fail(SBD_ERR_INVALID_ARG, "gumbel is not 16-byte aligned");
+  s = sbd::device_ready();
+  if (s != SBD_OK) return s;
   const sbd::HeadPlan p = sbd::head_plan(*desc);
   const size_t need = sbd::head_workspace_bytes(p);
   if (!workspace || workspace_bytes < need)
@@ -291,6 +322,8 @@ sbd_status select_call(int32_t rule, int32_t batch, int32_t block_k, const float
     if (!ptrs[i]) return fail(SBD_ERR_INVALID_ARG, "%s is NULL", names[i]);
   if (rule != SBD_SELECT_EB_ENTROPY && !confidence)
     return fail(SBD_ERR_INVALID_ARG, "confidence is NULL but rule %d orders by confidence", rule);
+  const sbd_status s = sbd::device_ready();
+  if (s != SBD_OK) return s;
   return sbd::select_launch(rule, batch, block_k, entropy, confidence, token, threshold, masked,
                             block_tokens, n_unmasked, (cudaStream_t)stream);
 }
@@ -374,6 +407,8 @@ sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w,
                 workspace ? workspace_bytes : (size_t)0);
   if (need > 0 && !aligned16(workspace))
     return fail(SBD_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+  s = sbd::device_ready();
+  if (s != SBD_OK) return s;
   return sbd::linear_launch(desc->rows, desc->in_features, desc->out_features, x, w, y,
                             workspace, (cudaStream_t)stream);
 }
@@ -386,6 +421,8 @@ sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t voc
   if (n_rows == 0 || vocab == 0) return SBD_OK;
   if (!row_ids) return fail(SBD_ERR_INVALID_ARG, "row_ids is NULL");
   if (!out) return fail(SBD_ERR_INVALID_ARG, "out is NULL");
+  const sbd_status s = sbd::device_ready();
+  if (s != SBD_OK) return s;
   return sbd::gumbel_fill_launch(n_rows, row_ids, vocab, seed, offset, out, (cudaStream_t)stream);
 }
 

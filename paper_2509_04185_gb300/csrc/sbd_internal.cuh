@@ -16,6 +16,10 @@ namespace sbd {
 sbd_status fail(sbd_status st, const char* fmt, ...);
 sbd_status cuda_fail(cudaError_t e, const char* what);
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// Queries the current device once (SM count, error-word address) and
+// fails with the reason recorded when that is impossible; every entry point
+// that launches calls it before num_sms() / device_error_word().
+sbd_status device_ready();
 int num_sms();                       // SMs of the current device (cached per device)
 int* device_error_word();            // device address of the error word (current device)
 
@@ -53,6 +57,9 @@ struct HeadPlan {
 };
 HeadPlan head_plan(const sbd_head_desc& d);
 size_t head_workspace_bytes(const HeadPlan& p);
+// A lower bound of head_workspace_bytes for a descriptor, with no device
+// query (the per-CTA partials of one CTA); 0 for an invalid descriptor.
+size_t head_workspace_floor(const sbd_head_desc& d);
 // Counter-based noise in place of a noise buffer (philox.cuh).
 struct PhiloxNoise {
   uint64_t seed, offset;

@@ -104,10 +104,12 @@ def test_full_size_configs(sbd, name):
     _run_and_compare(sbd, gen.get_workload(name), seed=0)
 
 
-def test_sweep_layer_k32(sbd):
-    """One layer of the 32-layer sweep at its largest block (k = 32: 128
-    packed rows per KV head), batch 16, cache 8192."""
-    _run_and_compare(sbd, gen.sweep_workload(32), seed=0)
+@pytest.mark.parametrize("k", [4, 8, 16, 32])
+def test_sweep_layer(sbd, k):
+    """One layer of the 32-layer sweep at each of its block sizes (k = 32:
+    128 packed rows per KV head; k = 4: 16, the register-accumulator
+    kernel), batch 16, cache 8192."""
+    _run_and_compare(sbd, gen.sweep_workload(k), seed=k)
 
 
 @pytest.mark.parametrize("k,L,splits", [(8, 8192, 0), (8, 8192, 13), (16, 4096, 0), (32, 2048, 3),

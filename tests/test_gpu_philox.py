@@ -44,7 +44,8 @@ def _case(B, k, V, H, dtype, seed):
 
 @pytest.mark.parametrize("B,k,V,H,dtype", [(1, 16, 4096 + 5, 512, "bf16"), (2, 16, 40000, 1024, "bf16"),
                                            (16, 32, 1500, 128, "bf16"), (3, 7, 777, 64, "bf16"),
-                                           (2, 8, 2000, 128, "f32")])
+                                           (2, 8, 2000, 128, "f32"),
+                                           (1, 16, 128256, 4096, "bf16")])
 @pytest.mark.parametrize("tau", [1.0, 0.3])
 def test_head_with_philox_noise(sbd, B, k, V, H, dtype, tau):
     import torch

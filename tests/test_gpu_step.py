@@ -7,7 +7,8 @@ import pytest
 
 import gen
 import oracle
-from tests.helpers import ENTROPY_TOL, compare_unmask, step_inputs, to_dev
+from tests.helpers import (ENTROPY_TOL, GAMMA_MARGIN, compare_unmask, step_inputs, to_dev,
+                           token_tolerance, top2_gap)
 
 pytestmark = pytest.mark.gpu
 
@@ -28,7 +29,8 @@ def _loop(sbd, w, gamma, seed=0, max_steps=None):
     masked = torch.from_numpy(d["masked"]).cuda()
     bt = torch.from_numpy(d["block_tokens"]).cuda()
     m_host = d["masked"].copy()
-    steps, exempt = 0, 0
+    bt_host = d["block_tokens"].copy()
+    steps, exempt, tok_exempt = 0, 0, 0
     while m_host.any():
         sbd.sbd_block_attention(att["q"], att["k_cache"], att["v_cache"], lens, att["k_blk"],
                                 att["v_blk"])
@@ -39,21 +41,39 @@ def _loop(sbd, w, gamma, seed=0, max_steps=None):
         n_un = sbd.sbd_eb_select(ent, tok, gamma, masked, bt)
         new_m = masked.cpu().numpy()
         # oracle on the same state
-        rent, rtok, _ = oracle.head_entropy_sample(oracle.widen(hidden, dt), d["w"], dt, m_host,
-                                                   gumbel, 1.0)
+        rent, rtok, zs = oracle.head_entropy_sample(oracle.widen(hidden, dt), d["w"], dt, m_host,
+                                                    gumbel, 1.0)
         e = ent.cpu().numpy()
+        t = tok.cpu().numpy()
         sel = m_host.astype(bool)
         assert np.abs(e[sel] - rent[sel]).max() <= ENTROPY_TOL
-        exempt += compare_unmask(m_host, rent, gamma, new_m, tie_tol=2 * ENTROPY_TOL)
+        # the order-tie rule of the comparison: oracle entropies closer
+        # than GAMMA_MARGIN may be taken in either order
+        exempt += compare_unmask(m_host, rent, gamma, new_m, tie_tol=GAMMA_MARGIN)
         nu = n_un.cpu().numpy()
         assert np.all(nu[m_host.any(axis=1)] >= 1)
         assert np.array_equal(nu, (m_host.astype(int) - new_m.astype(int)).sum(axis=1))
+        # committed tokens: the sampled token at exactly the newly unmasked
+        # positions, equal to the oracle's except at a score tie
+        bt_now = bt.cpu().numpy()
+        newly = sel & ~new_m.astype(bool)
+        assert np.array_equal(bt_now[newly], t[newly])
+        assert np.array_equal(bt_now[~newly], bt_host[~newly])
+        acc = w.hidden // (16 if dt == "bf16" else 1)
+        for b, i in zip(*np.nonzero(newly)):
+            if bt_now[b, i] != rtok[b, i]:
+                z = zs[(b, i)]
+                assert top2_gap(z, gumbel[b, i], 1.0) < token_tolerance(z, acc), (steps, b, i)
+                tok_exempt += 1
+        bt_host = bt_now
         m_host = new_m
         steps += 1
         assert steps <= w.block_k
     final = bt.cpu().numpy()
     assert (final >= 0).all() and (final < w.vocab).all()
     assert sbd.sbd_device_error() == 0
+    print(f"{w.name}: {steps} steps, unmask exemptions {exempt}, token exemptions {tok_exempt}")
+    assert tok_exempt <= 1
     return steps, exempt
 
 
