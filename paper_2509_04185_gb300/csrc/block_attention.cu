@@ -483,52 +483,86 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
   }
 }
 
-// Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.  One CTA per
-// (packed row, KV head, sequence); thread d owns output element d (D is 64
-// or 128, so whole warps take part).  The kernel is latency-bound: for each
-// group of 32 splits a thread requests its column of all of them, and lane s
-// the log-sum-exp of split s (shared through shuffles), before any is used,
-// so that one memory round trip covers the group; groups merge online.
-template <typename OutT>
-__global__ void __launch_bounds__(128)
+// Merge of the split partials: O = sum_s 2^(lse_s - lse) O_s.  One warp per
+// (packed row, KV head, sequence), kCombineRows rows per CTA: lane s holds
+// the log-sum-exp of split s, and each lane owns D / 32 consecutive output
+// columns.  The kernel is latency-bound: for each group of 32 splits a lane
+// requests the log-sum-exp and its columns of all of them before it uses
+// any, so that one memory round trip covers the group; groups merge online.
+// (One 128-thread CTA per row instead took 12.6 us for 2048 CTAs at 4
+// splits, its time growing with the CTA count.)
+constexpr int kCombineRows = 4;
+
+template <int D, typename OutT>
+__global__ void __launch_bounds__(32 * kCombineRows)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
-                    OutT* __restrict__ out, int k, int Hq, int Hkv, int G, int M, int D,
-                    int splits) {
-  constexpr int kGroup = 32;
+                    OutT* __restrict__ out, int k, int Hq, int Hkv, int G, int M, int splits) {
+  constexpr int kPer = D / 32;                 // columns per lane: 2 or 4
   grid_dependency_wait();
-  const int r = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
-  const int d = threadIdx.x, lane = threadIdx.x & 31;
-  if (d >= D) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kCombineRows + warp, hkv = blockIdx.y, b = blockIdx.z;
+  if (r >= M) return;
   const size_t pair = (size_t)b * Hkv + hkv;
   const float* lse = part_lse + pair * splits * M + r;
-  const float* po = part_o + (pair * splits * M + r) * D + d;
-  float mx = -INFINITY, sum = 0.f, acc = 0.f;
-  for (int s0 = 0; s0 < splits; s0 += kGroup) {
-    const float l_lane = s0 + lane < splits ? lse[(size_t)(s0 + lane) * M] : -INFINITY;
-    float v[kGroup];
+  const float* po = part_o + (pair * splits * M + r) * D + kPer * lane;
+  const size_t po_stride = (size_t)M * D;
+  float mx = -INFINITY, sum = 0.f, acc[kPer];
 #pragma unroll
-    for (int e = 0; e < kGroup; ++e) v[e] = s0 + e < splits ? po[(size_t)(s0 + e) * M * D] : 0.f;
+  for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
+  for (int s0 = 0; s0 < splits; s0 += 32) {
+    const int n = min(32, splits - s0);
+    const float l_lane = lane < n ? lse[(size_t)(s0 + lane) * M] : -INFINITY;
+    float v[32][kPer];
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      if (e < n) {
+        const float* src = po + (size_t)(s0 + e) * po_stride;
+        if constexpr (kPer == 4) {
+          const float4 x = *reinterpret_cast<const float4*>(src);
+          v[e][0] = x.x; v[e][1] = x.y; v[e][2] = x.z; v[e][3] = x.w;
+        } else {
+          const float2 x = *reinterpret_cast<const float2*>(src);
+          v[e][0] = x.x; v[e][1] = x.y;
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < kPer; ++c) v[e][c] = 0.f;
+      }
+    }
     const float gm = warp_max(l_lane);
     if (gm == -INFINITY) continue;               // every split of the group is empty
     if (gm > mx) {
       const float c = exp2f(mx - gm);            // 0 while mx = -inf
       sum *= c;
-      acc *= c;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) acc[e] *= c;
       mx = gm;
     }
 #pragma unroll
-    for (int e = 0; e < kGroup; ++e) {
-      const float wt = exp2f(__shfl_sync(0xffffffffu, l_lane, e) - mx);
+    for (int e = 0; e < 32; ++e) {
+      const float wt = exp2f(__shfl_sync(0xffffffffu, l_lane, e) - mx);   // 0 past n
       sum += wt;
-      if (wt > 0.f) acc = fmaf(wt, v[e], acc);
+      if (wt > 0.f) {
+#pragma unroll
+        for (int c = 0; c < kPer; ++c) acc[c] = fmaf(wt, v[e][c], acc[c]);
+      }
     }
   }
-  acc = sum > 0.f ? acc / sum : 0.f;
-  const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + d;
-  if constexpr (sizeof(OutT) == 2)
-    out[o] = __float2bfloat16_rn(acc);
-  else
-    out[o] = acc;
+  const float inv = sum > 0.f ? 1.f / sum : 0.f;
+  const size_t o = (((size_t)b * k + r / G) * Hq + hkv * G + r % G) * D + kPer * lane;
+  if constexpr (sizeof(OutT) == 2) {
+    if constexpr (kPer == 4) {
+      uint2 w;
+      w.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      w.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      *reinterpret_cast<uint2*>(out + o) = w;
+    } else {
+      *reinterpret_cast<uint32_t*>(out + o) = pack_bf16(acc[0] * inv, acc[1] * inv);
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < kPer; ++c) out[o + c] = acc[c] * inv;
+  }
 }
 
 // ------------------------------------------------------------ fp32 variant
@@ -774,11 +808,13 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
     const float* po = a.part_o;
     const float* pl = a.part_lse;
     __nv_bfloat16* o = (__nv_bfloat16*)out;
-    int k = p.k, Hq = p.Hq, Hkv = p.Hkv, G = p.G, M = p.M, D = p.D, S = p.splits;
+    int k = p.k, Hq = p.Hq, Hkv = p.Hkv, G = p.G, M = p.M, S = p.splits;
     void* args[] = {(void*)&po, (void*)&pl, (void*)&o, (void*)&k, (void*)&Hq, (void*)&Hkv,
-                    (void*)&G,  (void*)&M,  (void*)&D, (void*)&S};
-    s = launch_pdl((const void*)attn_combine_kernel<__nv_bfloat16>, dim3(p.M, p.Hkv, p.B),
-                   dim3(128), 0, st, args, "attn_combine_kernel launch");
+                    (void*)&G,  (void*)&M,  (void*)&S};
+    const void* fn = p.D == 128 ? (const void*)attn_combine_kernel<128, __nv_bfloat16>
+                                : (const void*)attn_combine_kernel<64, __nv_bfloat16>;
+    s = launch_pdl(fn, dim3((p.M + kCombineRows - 1) / kCombineRows, p.Hkv, p.B),
+                   dim3(32 * kCombineRows), 0, st, args, "attn_combine_kernel launch");
     if (s != SBD_OK) return s;
   }
   return SBD_OK;

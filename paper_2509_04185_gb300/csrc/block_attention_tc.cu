@@ -173,10 +173,20 @@ struct TcArgs {
 // lives in TMEM lane r, and the two warps of its lane quadrant take 64 of the
 // pair's 128 columns each (one tile each).  R = 2 (M <= 64): rows are also
 // copied to lanes 64 + r (the MMA pads to 128 rows anyway), so four warps on
-// all four SM sub-partitions share a row, 32 columns each.  R = 4 (M <= 32):
-// a copy in every lane quadrant, all eight warps share a row, 16 columns
-// each.  The warps sharing a row exchange their partial maxima through shared
-// memory at a named barrier and take identical decisions.
+// all four SM sub-partitions share a row, 32 columns each: copy 0 (lanes
+// 0-63) takes the pair's first tile, copy 1 (lanes 64-127) the second.  The
+// warps sharing a row exchange their partial maxima through shared memory at
+// a named barrier and take identical decisions.
+//
+// PV with R = 2.  A tcgen05.mma of M = 128 and K = 16 measured the same time
+// for every N up to 256 (~95 ns on GB300), so N = D leaves half of each
+// instruction idle.  Each copy of a row therefore accumulates its own tile
+// only: lane r of P holds the row's probabilities over the keys of its
+// copy's tile, and one instruction with B = [V of 16 keys of tile 0 | V of
+// the same 16 rows of tile 1] (N = 2 D) adds P_copy0 V_tile0 to columns
+// [0, D) and P_copy1 V_tile1 to columns [D, 2 D) of O (the other two blocks
+// of the product land in columns no lane reads).  4 instructions per pair
+// instead of 8; the two partial sums of a row are added in the epilogue.
 template <int D, int R>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
@@ -188,8 +198,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   constexpr int kKVSub = kTileKeys * 128;          // one tile's K or V sub-tile: 8 KB
   constexpr int kPairSub = 2 * kKVSub;             // a pair's K or V sub-tile: 16 KB
   constexpr int kPairBytes = 2 * kSub * kPairSub;  // K sub-tiles then V sub-tiles
-  constexpr uint32_t kTmemCols = 512;              // S0 | S1 (128 each) | O
+  constexpr uint32_t kTmemCols = 512;              // S0 | S1 (128 each) | O (R * D)
   constexpr uint32_t kOCol = 2 * kPairKeys;
+  static_assert(R == 1 || R == 2, "row copies");
+  static_assert(kOCol + R * D <= kTmemCols, "O fits the allocation");
   // With D = 128 the K region of a pair (32 KB) is exactly a P block, and K is
   // dead once S of the pair is computed: P is written there, and the ring gets
   // the shared memory separate P buffers would take.
@@ -214,16 +226,20 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const uint32_t q_s = sbase;                              // kSub x 16 KB
   const uint32_t p_s = q_s + kSub * kQBytes;               // 2 x 32 KB unless kPInK
   const uint32_t kv_s = p_s + (kPInK ? 0 : 4 * kQBytes);   // kPairs x kPairBytes
-  // Tile j of this split lives in pair slot (j / 2) mod kPairs, half j mod 2:
-  // the two tiles of a pair sit back to back in every sub-tile, so that a
-  // pair's keys form one 128-row operand.
+  // Tile j of this split lives in pair slot (j / 2) mod kPairs, half j mod 2.
+  // K: the two tiles of a pair sit back to back in every sub-tile, so that a
+  // pair's keys form one 128-row operand of S.  V: the sub-tiles are ordered
+  // (tile 0, columns 0-63), (tile 0, 64-127), (tile 1, 0-63), (tile 1,
+  // 64-127), 8 KB apart, so that the D columns of one tile, or of both tiles
+  // side by side, form one MN-major operand of PV with a constant stride.
   auto k_chunk = [&](int j, int h) -> uint32_t {
     return kv_s + ((j >> 1) % kPairs) * kPairBytes + h * kPairSub + (j & 1) * kKVSub;
   };
   auto v_chunk = [&](int j, int h) -> uint32_t {
-    return kv_s + ((j >> 1) % kPairs) * kPairBytes + (kSub + h) * kPairSub + (j & 1) * kKVSub;
+    return kv_s + ((j >> 1) % kPairs) * kPairBytes + kSub * kPairSub + ((j & 1) * kSub + h) * kKVSub;
   };
-  // P block of pair q: two 16 KB sub-tiles (keys 0-63, 64-127)
+  // P block of pair q: R = 1, two 16 KB sub-tiles (keys 0-63, 64-127); R = 2,
+  // one sub-tile whose row r holds lane r's keys (its copy's tile)
   auto p_block = [&](int q) -> uint32_t {
     return kPInK ? k_chunk(2 * q, 0) : p_s + (q & 1) * 2 * kQBytes;
   };
@@ -388,17 +404,31 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         tc_commit(&s_full[q & 1]);
       };
-      // O += P V over the pair's keys, 16 keys per instruction.
+      // O += P V over the pair's keys, 16 keys per instruction (R = 1), or
+      // 16 keys of each tile per instruction into the two copies' halves of
+      // O (R = 2; N = D only for a last pair of one tile, whose second copy
+      // has no keys).
       auto issue_pv = [&](int q) {
-        const int nk = 4 * min(2, n - 2 * q);
+        const int nt = min(2, n - 2 * q);
         const uint32_t pb = p_block(q);
         const uint32_t vb = v_chunk(2 * q, 0);
+        if constexpr (R == 1) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          if (kk >= nk) break;
-          const uint64_t ad = sw128_desc(pb + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
-          const uint64_t bd = sw128_desc(vb + kk * 16 * 128, kPairSub, 1024);
-          tc_mma(tmem + kOCol, ad, bd, id_o, (q > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk) {
+            if (kk >= 4 * nt) break;
+            const uint64_t ad = sw128_desc(pb + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
+            const uint64_t bd = sw128_desc(vb + (kk / 4) * kSub * kKVSub + (kk % 4) * 16 * 128,
+                                           kKVSub, 1024);
+            tc_mma(tmem + kOCol, ad, bd, id_o, (q > 0 || kk > 0) ? 1u : 0u);
+          }
+        } else {
+          const uint32_t id_pv = idesc_bf16(kRows, nt * D, true);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = sw128_desc(pb + kk * 32, 16, 1024);
+            const uint64_t bd = sw128_desc(vb + kk * 16 * 128, kKVSub, 1024);
+            tc_mma(tmem + kOCol, ad, bd, id_pv, (q > 0 || kk > 0) ? 1u : 0u);
+          }
         }
         tc_commit(&pv_done[q & 1]);
         tc_commit(&kv_empty[q % kPairs]);
@@ -429,8 +459,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
   } else {
     // ------------------------------------------------ softmax warps
-    static_assert(R == 1 || R == 2 || R == 4, "row copies");
-    constexpr int kCW = kPairKeys / (2 * R);     // columns per warp: 64, 32 or 16
+    constexpr int kCW = kPairKeys / (2 * R);     // columns per warp: 64 or 32
     constexpr int kQuadStride = 4 / R;           // lane quadrants between copies of a row
     constexpr int kRowsPerCopy = kRows / R;
     constexpr int kGroupThreads = 64 * R;        // the warps that share a row
@@ -439,11 +468,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int sub = sw >> 2;                     // 0 or 1 within the quadrant
     const int lane_t = quad * 32 + lane;         // TMEM lane
     const int row = lane_t % kRowsPerCopy;       // packed row
-    const int dup = lane_t / kRowsPerCopy;       // copy of the row (R = 2)
+    const int dup = lane_t / kRowsPerCopy;       // copy of the row (R = 2): its tile
     const int cbase = kCW * (dup * 2 + sub);     // this warp's columns of a pair
     const int half = cbase / kTileKeys;          // ... all inside one tile
     const int coff = cbase % kTileKeys;          // first column inside that tile
-    const bool owns_o = dup == 0;                // O row `row` lives in this lane
+    const bool owns_o = dup == 0;                // this lane writes row `row` out
+    // this lane's O: R = 1 the row's, R = 2 its copy's partial (own tile)
+    const uint32_t o_col = kOCol + (uint32_t)(dup * D);
     const int bar_id = 1 + quad % kQuadStride;  // one named barrier per row group
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     // softmax warp index of (quadrant q, sub s)
@@ -540,7 +571,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       // The P block of this pair is free once PV(q-2) is done (it lives in
       // the pair's own K sub-tiles for D = 128); O itself is only touched
       // (rescaled) after PV(q-1).
-      const int wait_q = (warp_rescale && owns_o) ? q - 1 : (kPInK ? -1 : q - 2);
+      const int wait_q = warp_rescale ? q - 1 : (kPInK ? -1 : q - 2);
       bool waited = wait_q < 0 || mbar_wait(&pv_done[wait_q & 1], (wait_q >> 1) & 1, a.err);
       if (!__all_sync(0xffffffffu, waited)) {
         ok = false;
@@ -554,23 +585,24 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         l *= alpha;
         m_ref = mt;
       }
-      if (warp_rescale && owns_o) {
-        // the two sub-warps of the rows' own quadrant rescale half of O each
+      if (warp_rescale) {
+        // the two sub-warps of a quadrant rescale half of its lanes' O each
 #pragma unroll
         for (int c = sub * (D / 32); c < (sub + 1) * (D / 32); ++c) {
           uint32_t r[16];
-          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_ld16(tmem + lane_addr + o_col + c * 16, r);
           tc_wait_ld();
 #pragma unroll
           for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-          tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_st16(tmem + lane_addr + o_col + c * 16, r);
         }
         tc_wait_st();
       }
       // P = 2^(scale * s - m_ref) as bf16 into this warp's columns of the
-      // pair's P block (row `row`).  Rows past M and, with R = 2, rows 64+
-      // of P are never written: their O rows are garbage that is never read.
-      const uint32_t pb = p_block(q) + half * kQBytes;
+      // pair's P block, in row `lane_t` (R = 1: the packed row; R = 2: the
+      // copy's row, whose keys are its tile's).  Rows past M are garbage
+      // whose O rows are never read.
+      const uint32_t pb = p_block(q) + (R == 1 ? half * kQBytes : 0);
       {
         const float nm = -m_ref;
         float psum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -582,7 +614,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
             p[e] = exp2f(fmaf(s[c * 8 + e], a.scale_log2, nm));
             psum[e] += p[e];
           }
-          st_shared_v4(swz(pb, row, coff / 8 + c),
+          st_shared_v4(swz(pb, lane_t, coff / 8 + c),
                        make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7])));
         }
@@ -609,12 +641,45 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       for (int s2 = 0; s2 < 2; ++s2)
         lsum += red_l[sw_of(quad_of(d2), s2) * 32 + lane];
     const bool mine = owns_o && row < a.M;
-    // the two sub-warps of the row's quadrant write half of the D columns each
+    // the two sub-warps of a quadrant take half of the D columns each
     const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
-    bool final_ok =
-        ok && np > 0 && owns_o && mbar_wait(&pv_done[(np - 1) & 1], ((np - 1) >> 1) & 1, a.err);
+    bool final_ok = ok && np > 0 && mbar_wait(&pv_done[(np - 1) & 1], ((np - 1) >> 1) & 1, a.err);
     final_ok = __all_sync(0xffffffffu, final_ok);   // the reads below are warp-collective
-    if (final_ok) {
+    // R = 2: copy 1 hands its partial O to copy 0 through shared memory (the
+    // ring, idle once the last PV is done: every load was consumed by an
+    // MMA before it).  A split of one tile gave copy 1 no keys; its half of
+    // O was never written and is left out.
+    constexpr int kStageStride = D + 1;           // floats per staged row (bank spread)
+    float* stage = reinterpret_cast<float*>(smem_raw + (kv_s - smem_u32(smem_raw)));
+    const bool has_copy1 = R == 2 && n >= 2;
+    if constexpr (R == 2) {
+      if (final_ok && dup == 1 && has_copy1) {
+        tc_fence_after();
+#pragma unroll
+        for (int c = c_lo; c < c_hi; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + o_col + c * 16, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) stage[row * kStageStride + c * 16 + e] = __uint_as_float(r[e]);
+        }
+      }
+      asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(kGroupThreads) : "memory");
+    }
+    // Row `row` of O in columns [16 c, 16 c + 16): this lane's accumulator
+    // plus, with R = 2, the other copy's.
+    auto load_o = [&](int c, float (&o)[16]) {
+      uint32_t r[16];
+      tc_ld16(tmem + lane_addr + o_col + c * 16, r);
+      tc_wait_ld();
+#pragma unroll
+      for (int e = 0; e < 16; ++e) o[e] = __uint_as_float(r[e]);
+      if (has_copy1) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) o[e] += stage[row * kStageStride + c * 16 + e];
+      }
+    };
+    if (final_ok && owns_o) {
       tc_fence_after();
       const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
       if (a.splits == 1) {
@@ -623,19 +688,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                  : nullptr;
 #pragma unroll
         for (int c = c_lo; c < c_hi; ++c) {
-          uint32_t r[16];
-          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
-          tc_wait_ld();
+          float o[16];
+          load_o(c, o);
           if (mine) {
             uint4 w0, w1;
-            w0.x = pack_bf16(__uint_as_float(r[0]) * inv, __uint_as_float(r[1]) * inv);
-            w0.y = pack_bf16(__uint_as_float(r[2]) * inv, __uint_as_float(r[3]) * inv);
-            w0.z = pack_bf16(__uint_as_float(r[4]) * inv, __uint_as_float(r[5]) * inv);
-            w0.w = pack_bf16(__uint_as_float(r[6]) * inv, __uint_as_float(r[7]) * inv);
-            w1.x = pack_bf16(__uint_as_float(r[8]) * inv, __uint_as_float(r[9]) * inv);
-            w1.y = pack_bf16(__uint_as_float(r[10]) * inv, __uint_as_float(r[11]) * inv);
-            w1.z = pack_bf16(__uint_as_float(r[12]) * inv, __uint_as_float(r[13]) * inv);
-            w1.w = pack_bf16(__uint_as_float(r[14]) * inv, __uint_as_float(r[15]) * inv);
+            w0.x = pack_bf16(o[0] * inv, o[1] * inv);
+            w0.y = pack_bf16(o[2] * inv, o[3] * inv);
+            w0.z = pack_bf16(o[4] * inv, o[5] * inv);
+            w0.w = pack_bf16(o[6] * inv, o[7] * inv);
+            w1.x = pack_bf16(o[8] * inv, o[9] * inv);
+            w1.y = pack_bf16(o[10] * inv, o[11] * inv);
+            w1.z = pack_bf16(o[12] * inv, o[13] * inv);
+            w1.w = pack_bf16(o[14] * inv, o[15] * inv);
             *reinterpret_cast<uint4*>(dst + c * 16) = w0;
             *reinterpret_cast<uint4*>(dst + c * 16 + 8) = w1;
           }
@@ -645,15 +709,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         float* dst = mine ? a.part_o + prow * D : nullptr;
 #pragma unroll
         for (int c = c_lo; c < c_hi; ++c) {
-          uint32_t r[16];
-          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
-          tc_wait_ld();
+          float o[16];
+          load_o(c, o);
           if (mine) {
 #pragma unroll
             for (int e = 0; e < 16; e += 4)
               *reinterpret_cast<float4*>(dst + c * 16 + e) =
-                  make_float4(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv,
-                              __uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
+                  make_float4(o[e] * inv, o[e + 1] * inv, o[e + 2] * inv, o[e + 3] * inv);
           }
         }
         if (mine && sub == 0) a.part_lse[prow] = lsum > 0.f ? m_ref + log2f(lsum) : -INFINITY;
@@ -712,15 +774,13 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t smem = attn_tc_smem_bytes(p.D);
-  // copies of every packed row in the 128 MMA rows: 4, 2 or 1
-  const int R = p.M <= kRows / 4 ? 4 : (p.M <= kRows / 2 ? 2 : 1);
+  // copies of every packed row in the 128 MMA rows: 2 or 1
+  const int R = p.M <= kRows / 2 ? 2 : 1;
   const void* fn;
   if (p.D == 128)
-    fn = R == 4 ? (const void*)attn_tc_kernel<128, 4>
-                : (R == 2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>);
+    fn = R == 2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>;
   else
-    fn = R == 4 ? (const void*)attn_tc_kernel<64, 4>
-                : (R == 2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>);
+    fn = R == 2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
   // The block keys/values [B, k, Hkv, D] as 4-D tensors (D, Hkv, k, B), read
