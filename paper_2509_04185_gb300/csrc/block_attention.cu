@@ -684,6 +684,26 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
   } else {
     p.splits = choose_splits(p.B * p.Hkv, tiles, num_sms());
   }
+  // tcgen05 path: the splits of a (sequence, KV head) merge in shared memory
+  // as one thread-block cluster (at most 16 CTAs) when the device can hold
+  // all the clusters at once.  An automatic split count is lowered, down to
+  // 3/5 of it, to the largest cluster size that fits (GB300, one 227 KB CTA
+  // per SM: 36 clusters of 4, 15 of 8, 7 of 16); at batch 1, Llama-8B, 4096
+  // cached keys, 12 splits in clusters took 12.9 us against 13.9 us for 19
+  // splits merged by attn_combine_kernel.  Otherwise the partials go through
+  // the workspace and attn_combine_kernel.
+  p.cluster = false;
+  if (p.bf16 && p.M >= kTcMinRows && p.B > 0 && p.splits >= 2) {
+    const int hi = p.splits < 16 ? p.splits : 16;
+    const int lo = d.num_splits > 0 ? p.splits : (3 * p.splits + 4) / 5;
+    for (int s = hi; s >= lo && s >= 2; --s) {
+      if (attn_tc_cluster_ok(p, s)) {
+        p.splits = s;
+        p.cluster = true;
+        break;
+      }
+    }
+  }
   // With more CTAs than one wave, the CTAs take the sequences longest first
   // (the pick costs B^2 comparisons per CTA, hence the batch limit).
   p.order = p.bf16 && p.B > 1 && p.B <= kOrderMaxB &&
@@ -701,7 +721,7 @@ AttnPlan attn_plan(const sbd_attn_desc& d) {
 }
 
 size_t attn_workspace_bytes(const AttnPlan& p) {
-  if (p.splits <= 1) return 0;
+  if (p.splits <= 1 || p.cluster) return 0;
   const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
   return align_up(n * p.D * sizeof(float), 256) + align_up(n * sizeof(float), 256);
 }
@@ -771,8 +791,9 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   const size_t n = (size_t)p.B * p.Hkv * p.splits * p.M;
-  a.part_o = (float*)ws;
-  a.part_lse = p.splits > 1 ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
+  const bool use_ws = p.splits > 1 && !p.cluster;
+  a.part_o = use_ws ? (float*)ws : nullptr;
+  a.part_lse = use_ws ? (float*)((char*)ws + align_up(n * p.D * sizeof(float), 256)) : nullptr;
 
   // Up to 16 packed rows the mma.sync kernel measures faster (the tcgen05
   // kernel pads every tile to 128 rows); from 17 on, tcgen05, with every row
@@ -804,7 +825,7 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
     if (s != SBD_OK) return s;
   }
   }
-  if (p.splits > 1) {
+  if (use_ws) {
     const float* po = a.part_o;
     const float* pl = a.part_lse;
     __nv_bfloat16* o = (__nv_bfloat16*)out;

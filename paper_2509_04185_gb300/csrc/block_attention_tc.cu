@@ -37,6 +37,8 @@
 // (one split) or the split partial and its log-sum-exp.
 #include <math.h>
 
+#include <mutex>
+
 #include "sbd_internal.cuh"
 
 namespace {
@@ -129,6 +131,42 @@ __device__ __forceinline__ uint32_t idesc_bf16(int M, int N, bool b_mn) {
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// ------------------------------------------------------------ clusters
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The address of this CTA's shared-memory location `addr` in CTA `rank` of
+// the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_cluster_v4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ float2 ld_cluster_v2(uint32_t addr) {
+  float2 v;
+  asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr) : "memory");
+  return v;
+}
+
 // Address of (row, 16-byte chunk c) inside a [rows x 128 B] swizzled tile.
 __device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk) {
   return base + row * 128 + (((chunk ^ (row & 7)) & 7) << 4);
@@ -166,6 +204,8 @@ struct TcArgs {
   __nv_bfloat16* vc_app;
   int B, k, Hq, Hkv, G, M, Lmax, splits, n_causal;
   int order;                 // blockIdx.z -> sequence by descending length
+  int cluster;               // the splits of a (sequence, KV head) form one cluster and
+                             // merge their partials in shared memory (no part_o / part_lse)
   float scale_log2;
 };
 
@@ -652,6 +692,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     constexpr int kStageStride = D + 1;           // floats per staged row (bank spread)
     float* stage = reinterpret_cast<float*>(smem_raw + (kv_s - smem_u32(smem_raw)));
     const bool has_copy1 = R == 2 && n >= 2;
+    // Cluster merge: this CTA's normalised partial rows and their log2-sum-
+    // exps, 64 KB into the ring (past the copy-1 stage), read by every CTA of
+    // the cluster after a cluster barrier.
+    constexpr int kCStride = D + 4;             // floats per partial row (16-byte rows)
+    float* cpart = reinterpret_cast<float*>(smem_raw + (kv_s + 65536u - smem_u32(smem_raw)));
+    float* clse = cpart + kRows * kCStride;
     if constexpr (R == 2) {
       if (final_ok && dup == 1 && has_copy1) {
         tc_fence_after();
@@ -706,7 +752,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       } else {
         const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
-        float* dst = mine ? a.part_o + prow * D : nullptr;
+        float* dst = mine ? (a.cluster ? cpart + row * kCStride : a.part_o + prow * D) : nullptr;
 #pragma unroll
         for (int c = c_lo; c < c_hi; ++c) {
           float o[16];
@@ -718,13 +764,19 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                   make_float4(o[e] * inv, o[e + 1] * inv, o[e + 2] * inv, o[e + 3] * inv);
           }
         }
-        if (mine && sub == 0) a.part_lse[prow] = lsum > 0.f ? m_ref + log2f(lsum) : -INFINITY;
+        if (mine && sub == 0) {
+          const float lse = lsum > 0.f ? m_ref + log2f(lsum) : -INFINITY;
+          if (a.cluster) clse[row] = lse; else a.part_lse[prow] = lse;
+        }
       }
     } else if (n == 0 && a.splits > 1 && mine) {
       // an empty split contributes nothing
       const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
-      for (int d = c_lo * 16; d < c_hi * 16; ++d) a.part_o[prow * D + d] = 0.f;
-      if (sub == 0) a.part_lse[prow] = -INFINITY;
+      float* dst = a.cluster ? cpart + row * kCStride : a.part_o + prow * D;
+      for (int d = c_lo * 16; d < c_hi * 16; ++d) dst[d] = 0.f;
+      if (sub == 0) {
+        if (a.cluster) clse[row] = -INFINITY; else a.part_lse[prow] = -INFINITY;
+      }
     }
   }
   tc_fence_before();
@@ -732,6 +784,69 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   if (warp == 1) {
     tc_fence_after();
     tc_dealloc(tmem, kTmemCols);
+  }
+  if (a.cluster) {
+    // ------------------------------------------------ merge in the cluster
+    // The CTAs of a cluster are the splits of one (sequence, KV head).  After
+    // a cluster barrier every CTA's partial rows are visible to the others;
+    // CTA `rank` merges rows rank, rank + S, ... (one softmax warp a row,
+    // lane s reading split s's log2-sum-exp, D / 32 columns a lane) and
+    // writes them out; a second barrier keeps every CTA's shared memory
+    // alive until the others have read it.  All threads of every CTA reach
+    // both barriers: no role leaves the kernel early, and every wait before
+    // them is bounded.
+    cluster_sync_all();
+    if (warp >= 2) {
+      constexpr int kCStride = D + 4;
+      constexpr int kPer = D / 32;
+      const uint32_t cpart_s = kv_s + 65536u;
+      const uint32_t clse_s = cpart_s + (uint32_t)(kRows * kCStride * 4);
+      const int S = a.splits;
+      const int rank = (int)cluster_ctarank();
+      for (int r = rank + S * (warp - 2); r < a.M; r += S * kSoftWarps) {
+        const float l = lane < S ? ld_cluster_f32(mapa_shared(clse_s + 4u * r, lane)) : -INFINITY;
+        const float gm = warp_max(l);
+        const float w = (lane < S && gm != -INFINITY) ? exp2f(l - gm) : 0.f;
+        const float wsum = warp_sum(w);
+        float v[16][kPer];
+#pragma unroll
+        for (int s2 = 0; s2 < 16; ++s2) {
+          if (s2 < S) {
+            const uint32_t src = mapa_shared(cpart_s + 4u * (r * kCStride + kPer * lane), s2);
+            if constexpr (kPer == 4) {
+              const float4 x = ld_cluster_v4(src);
+              v[s2][0] = x.x; v[s2][1] = x.y; v[s2][2] = x.z; v[s2][3] = x.w;
+            } else {
+              const float2 x = ld_cluster_v2(src);
+              v[s2][0] = x.x; v[s2][1] = x.y;
+            }
+          }
+        }
+        float acc[kPer];
+#pragma unroll
+        for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
+#pragma unroll
+        for (int s2 = 0; s2 < 16; ++s2) {
+          const float ws = __shfl_sync(0xffffffffu, w, s2);    // 0 past S
+          if (s2 < S && ws > 0.f) {
+#pragma unroll
+            for (int c = 0; c < kPer; ++c) acc[c] = fmaf(ws, v[s2][c], acc[c]);
+          }
+        }
+        const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+        __nv_bfloat16* dst =
+            a.out + (((size_t)b * a.k + r / a.G) * a.Hq + hkv * a.G + r % a.G) * D + kPer * lane;
+        if constexpr (kPer == 4) {
+          uint2 o2;
+          o2.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+          o2.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+          *reinterpret_cast<uint2*>(dst) = o2;
+        } else {
+          *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
+        }
+      }
+    }
+    cluster_sync_all();
   }
 }
 
@@ -745,6 +860,50 @@ size_t attn_tc_smem_bytes(int D) {
   const int pairs = p_in_k ? 3 : 4;
   return 1024 + (size_t)sub * kRows * 128 + (p_in_k ? 0 : 4 * kRows * 128) +
          (size_t)pairs * 2 * sub * kPairKeys * 128;
+}
+
+// The kernel instance for head dimension D and M packed rows (copies of
+// every row in the 128 MMA rows: 2 up to 64 rows, else 1).
+static const void* attn_tc_fn(int D, int M) {
+  const bool two = M <= kRows / 2;
+  if (D == 128)
+    return two ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>;
+  return two ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>;
+}
+
+bool attn_tc_cluster_ok(const AttnPlan& p, int splits) {
+  // Whether every (sequence, KV head)'s `splits` CTAs can run as one cluster,
+  // all clusters at once.  The device's answer per (device, kernel, cluster
+  // size) is kept; the call is on every launch's host path.
+  struct Entry {
+    int dev;
+    const void* fn;
+    int splits;
+    int clusters;
+  };
+  static std::mutex mu;
+  static Entry cache[32];
+  static int n_cache = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  const void* fn = attn_tc_fn(p.D, p.M);
+  int clusters = -1;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < n_cache; ++i)
+      if (cache[i].dev == dev && cache[i].fn == fn && cache[i].splits == splits)
+        clusters = cache[i].clusters;
+  }
+  if (clusters < 0) {
+    clusters = max_active_clusters(fn, dim3(splits, p.Hkv, p.B), dim3(kThreads),
+                                   attn_tc_smem_bytes(p.D), splits);
+    std::lock_guard<std::mutex> lock(mu);
+    if (n_cache < 32) cache[n_cache++] = Entry{dev, fn, splits, clusters};
+  }
+  return (long long)clusters >= (long long)p.B * p.Hkv;
 }
 
 sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
@@ -773,14 +932,9 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.kc_app = (__nv_bfloat16*)kc_app;
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
+  a.cluster = p.cluster ? 1 : 0;
   const size_t smem = attn_tc_smem_bytes(p.D);
-  // copies of every packed row in the 128 MMA rows: 2 or 1
-  const int R = p.M <= kRows / 2 ? 2 : 1;
-  const void* fn;
-  if (p.D == 128)
-    fn = R == 2 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>;
-  else
-    fn = R == 2 ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>;
+  const void* fn = attn_tc_fn(p.D, p.M);
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
   // The block keys/values [B, k, Hkv, D] as 4-D tensors (D, Hkv, k, B), read
@@ -802,7 +956,7 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   CUtensorMap k_map = tk, v_map = tv;
   void* args[] = {(void*)&k_map, (void*)&v_map, (void*)&kb_map, (void*)&vb_map, (void*)&a};
   return launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(kThreads), smem, st, args,
-                    "attn_tc_kernel launch");
+                    "attn_tc_kernel launch", p.cluster ? p.splits : 1);
 }
 
 }  // namespace sbd

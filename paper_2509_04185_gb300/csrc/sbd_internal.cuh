@@ -33,6 +33,7 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
 struct AttnPlan {
   int B, k, Hq, Hkv, G, D, Lmax, M, splits, stages, MT, KG;
   bool order;         // CTAs take sequences longest first (more than one wave)
+  bool cluster;       // the splits of a (sequence, KV head) merge in a cluster (tcgen05 path)
   int n_causal;       // block rows i < n_causal see block keys j <= i only
   float scale_log2;   // softmax scale * log2(e)
   bool bf16;
@@ -46,6 +47,9 @@ sbd_status attn_launch(const AttnPlan& p, const void* q, const void* kc, const v
                        void* ws, void* kc_app, void* vc_app, cudaStream_t st);
 
 size_t attn_tc_smem_bytes(int D);
+// Whether the tcgen05 attention kernel can run the `splits` CTAs of every
+// (sequence, KV head) of plan p as one thread-block cluster, all at once.
+bool attn_tc_cluster_ok(const AttnPlan& p, int splits);
 sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtensorMap& tv,
                           const void* q, const int32_t* lens, const void* kb, const void* vb,
                           void* out, float* part_o, float* part_lse, void* kc_app,
@@ -88,8 +92,14 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Launch with programmatic dependent launch allowed: the kernel may be
 // scheduled while its predecessor on the stream finishes; every library
 // kernel calls griddepcontrol.wait before it touches global memory.
+// cluster_x > 1: CTAs of consecutive blockIdx.x form thread-block clusters of
+// that size.
 sbd_status launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
-                      void** args, const char* what);
+                      void** args, const char* what, int cluster_x = 1);
+// How many clusters of cluster_x CTAs (with `smem` bytes of dynamic shared
+// memory each) the current device can hold at once; 0 when the shape cannot
+// be launched as clusters.
+int max_active_clusters(const void* fn, dim3 grid, dim3 block, size_t smem, int cluster_x);
 
 }  // namespace sbd
 
