@@ -81,6 +81,17 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// The same with the A operand read from tensor memory (M = 128 lanes, K
+// packed as bf16 pairs along the columns).
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 __device__ __forceinline__ void tc_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -208,6 +219,72 @@ struct TcArgs {
                              // merge their partials in shared memory (no part_o / part_lse)
   float scale_log2;
 };
+
+// ------------------------------------------------ merge in the cluster
+// The CTAs of a cluster are the splits of one (sequence, KV head), each
+// holding its normalised partial rows (cpart_s: kRows x (D + 4) floats) and
+// their log2-sum-exps (after them) in shared memory.  After a cluster
+// barrier every CTA's partials are visible to the others; CTA `rank` merges
+// rows rank, rank + S, ... (softmax warp sw takes one row at a time, lane s
+// reading split s's log2-sum-exp, D / 32 columns a lane) and writes them
+// out; a second barrier keeps every CTA's shared memory alive until the
+// others have read it.  All threads of every CTA reach both barriers: no
+// role leaves the kernel early, and every wait before them is bounded.
+template <int D>
+__device__ __forceinline__ void cluster_merge(const TcArgs& a, int b, int hkv, uint32_t cpart_s,
+                                              int sw, int lane) {
+  cluster_sync_all();
+  if (sw >= 0 && sw < kSoftWarps) {
+    constexpr int kCStride = D + 4;
+    constexpr int kPer = D / 32;
+    const uint32_t clse_s = cpart_s + (uint32_t)(kRows * kCStride * 4);
+    const int S = a.splits;
+    const int rank = (int)cluster_ctarank();
+    for (int r = rank + S * sw; r < a.M; r += S * kSoftWarps) {
+      const float l = lane < S ? ld_cluster_f32(mapa_shared(clse_s + 4u * r, lane)) : -INFINITY;
+      const float gm = warp_max(l);
+      const float w = (lane < S && gm != -INFINITY) ? exp2f(l - gm) : 0.f;
+      const float wsum = warp_sum(w);
+      float v[16][kPer];
+#pragma unroll
+      for (int s2 = 0; s2 < 16; ++s2) {
+        if (s2 < S) {
+          const uint32_t src = mapa_shared(cpart_s + 4u * (r * kCStride + kPer * lane), s2);
+          if constexpr (kPer == 4) {
+            const float4 x = ld_cluster_v4(src);
+            v[s2][0] = x.x; v[s2][1] = x.y; v[s2][2] = x.z; v[s2][3] = x.w;
+          } else {
+            const float2 x = ld_cluster_v2(src);
+            v[s2][0] = x.x; v[s2][1] = x.y;
+          }
+        }
+      }
+      float acc[kPer];
+#pragma unroll
+      for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
+#pragma unroll
+      for (int s2 = 0; s2 < 16; ++s2) {
+        const float ws = __shfl_sync(0xffffffffu, w, s2);    // 0 past S
+        if (s2 < S && ws > 0.f) {
+#pragma unroll
+          for (int c = 0; c < kPer; ++c) acc[c] = fmaf(ws, v[s2][c], acc[c]);
+        }
+      }
+      const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+      __nv_bfloat16* dst =
+          a.out + (((size_t)b * a.k + r / a.G) * a.Hq + hkv * a.G + r % a.G) * D + kPer * lane;
+      if constexpr (kPer == 4) {
+        uint2 o2;
+        o2.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+        o2.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+        *reinterpret_cast<uint2*>(dst) = o2;
+      } else {
+        *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
+      }
+    }
+  }
+  cluster_sync_all();
+}
 
 // Softmax work split over the 128 columns of a pair.  R = 1: packed row r
 // lives in TMEM lane r, and the two warps of its lane quadrant take 64 of the
@@ -785,69 +862,507 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     tc_fence_after();
     tc_dealloc(tmem, kTmemCols);
   }
-  if (a.cluster) {
-    // ------------------------------------------------ merge in the cluster
-    // The CTAs of a cluster are the splits of one (sequence, KV head).  After
-    // a cluster barrier every CTA's partial rows are visible to the others;
-    // CTA `rank` merges rows rank, rank + S, ... (one softmax warp a row,
-    // lane s reading split s's log2-sum-exp, D / 32 columns a lane) and
-    // writes them out; a second barrier keeps every CTA's shared memory
-    // alive until the others have read it.  All threads of every CTA reach
-    // both barriers: no role leaves the kernel early, and every wait before
-    // them is bounded.
-    cluster_sync_all();
-    if (warp >= 2) {
-      constexpr int kCStride = D + 4;
-      constexpr int kPer = D / 32;
-      const uint32_t cpart_s = kv_s + 65536u;
-      const uint32_t clse_s = cpart_s + (uint32_t)(kRows * kCStride * 4);
-      const int S = a.splits;
-      const int rank = (int)cluster_ctarank();
-      for (int r = rank + S * (warp - 2); r < a.M; r += S * kSoftWarps) {
-        const float l = lane < S ? ld_cluster_f32(mapa_shared(clse_s + 4u * r, lane)) : -INFINITY;
-        const float gm = warp_max(l);
-        const float w = (lane < S && gm != -INFINITY) ? exp2f(l - gm) : 0.f;
-        const float wsum = warp_sum(w);
-        float v[16][kPer];
+  if (a.cluster) cluster_merge<D>(a, b, hkv, kv_s + 65536u, warp - 2, lane);
+}
+
+// ------------------------------------------------------------ wide row tiles
+// More than 64 packed rows (M = 65..128, e.g. k = 32 with 4 query heads per
+// KV head): every TMEM lane holds a distinct row, so the copy scheme of
+// attn_tc_kernel has nothing to pair, and PV needs D / 16 ... keys / 16
+// instructions of N = D.  What can still shrink is the score product and
+// the ring's hold on K.  Keys go in triples of 64-key tiles:
+//
+//   S_t = Q K_t^T     A = Q (shared, K-major), B = the triple's K (shared,
+//                     K-major), N = 192: D / 16 instructions per 192 keys
+//                     instead of per 128;
+//   O  += P_t V_t     A = P_t from tensor memory (tcgen05.mma with the A
+//                     operand in TMEM; bf16 pairs written by the softmax
+//                     warps with tcgen05.st), B = each tile's V (shared,
+//                     MN-major), N = D: 12 instructions per triple.
+//
+// Tensor memory: S 192 | O D | P 2 x 96 columns.  With P there, shared
+// memory holds Q and two separate rings: 2 triples of K, each freed as soon
+// as its score product is done, and V tiles, each freed after its PV
+// instructions.  S is a single buffer (S_{t+1} is issued once the softmax
+// warps hold S_t in registers); P is double-buffered, so that the
+// exponentials of triple t + 1 do not wait for PV_t.
+//
+// Warp roles: warp 0 loads K (TMA), warp 1 owns the tensor memory and
+// issues the MMAs, warp 2 loads V (TMA; zeroes value rows past the cache
+// length; copies the causal rows into the cache), warps 3-10 are the softmax
+// (two per lane quadrant, 96 of a triple's 192 columns each, the row maximum
+// agreed through shared memory).  Rescale rule, epilogue and cluster merge
+// as in attn_tc_kernel.
+constexpr int kTriTiles = 3;
+constexpr int kTriKeys = kTriTiles * kTileKeys;          // 192
+constexpr int kWideKSlots = 2;                           // K triples in the ring
+// V tiles in the ring: what is left of the 227 KB next to Q and the K ring
+template <int D> __host__ __device__ constexpr int wide_v_slots() { return D == 128 ? 6 : 8; }
+constexpr int kWideThreads = 96 + 32 * kSoftWarps;       // K, MMA, V, softmax warps
+
+__host__ __device__ constexpr int wide_tmem_o() { return kTriKeys; }              // 192
+template <int D> __host__ __device__ constexpr int wide_tmem_p() { return kTriKeys + D; }
+
+template <int D>
+__global__ void __launch_bounds__(kWideThreads, 1)
+attn_wide_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                 const __grid_constant__ CUtensorMap tmap_v,
+                 const __grid_constant__ CUtensorMap tmap_kb,
+                 const __grid_constant__ CUtensorMap tmap_vb, const TcArgs a) {
+  constexpr int kSub = D / 64;                     // 128-B column sub-tiles of a key row
+  constexpr int kKVSub = kTileKeys * 128;          // one tile's K or V sub-tile: 8 KB
+  constexpr int kTriSub = kTriTiles * kKVSub;      // a triple's K sub-tile: 24 KB
+  constexpr int kKSlotBytes = kSub * kTriSub;
+  constexpr int kVSlotBytes = kSub * kKVSub;
+  constexpr int kVSlots = wide_v_slots<D>();
+  constexpr int kQBytes = kRows * 128;             // one Q sub-tile: 16 KB
+  constexpr uint32_t kTmemCols = 512;
+  constexpr uint32_t kOCol = wide_tmem_o();
+  constexpr uint32_t kPCol = wide_tmem_p<D>();
+  constexpr uint32_t kPStride = kTriKeys / 2;      // columns of one P buffer
+  static_assert(kPCol + 2 * kPStride <= kTmemCols, "S, O and two P buffers fit the allocation");
+  constexpr int kCW = kTriKeys / 2;                // columns per softmax warp: 96
+
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t k_full[kWideKSlots], k_empty[kWideKSlots];
+  __shared__ __align__(8) uint64_t v_full[kVSlots], v_empty[kVSlots];
+  __shared__ __align__(8) uint64_t s_full, s_free, p_full[2], pv_done[2], q_ready, tail_bar;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ __align__(16) uint32_t red_buf[kSoftWarps * 32];
+  uint16_t* red_max = reinterpret_cast<uint16_t*>(red_buf);
+  float* red_l = reinterpret_cast<float*>(red_buf);
+  __shared__ int b_pick;
+
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t q_s = sbase;                                   // kSub x 16 KB
+  const uint32_t k_s = q_s + kSub * kQBytes;                    // kWideKSlots x kKSlotBytes
+  const uint32_t v_s = k_s + kWideKSlots * kKSlotBytes;         // kVSlots x kVSlotBytes
+  // tile j of the split: K in triple slot (j / 3) mod 2, position j mod 3 of
+  // every sub-tile (the triple's keys form one 192-row operand); V in tile
+  // slot j mod kVSlots
+  auto k_chunk = [&](int j, int h) -> uint32_t {
+    return k_s + ((j / kTriTiles) % kWideKSlots) * kKSlotBytes + h * kTriSub + (j % kTriTiles) * kKVSub;
+  };
+  auto v_chunk = [&](int j, int h) -> uint32_t {
+    return v_s + (j % kVSlots) * kVSlotBytes + h * kKVSub;
+  };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, hkv = blockIdx.y;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kWideKSlots; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < kVSlots; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    mbar_init(&s_full, 1);
+    mbar_init(&s_free, kSoftWarps);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&p_full[i], kSoftWarps);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(&q_ready, kSoftWarps);
+    mbar_init(&tail_bar, 1);
+    fence_mbar_init();
+  }
+  grid_dependency_wait();
+  if (a.order) {
+    longest_first_pick(a.lens, a.B, a.Lmax, blockIdx.z, &b_pick);
+    __syncthreads();
+  }
+  const int b = a.order ? b_pick : (int)blockIdx.z;
+  if (warp == 1) tc_alloc(&tmem_base_sh, kTmemCols);
+
+  int len = a.lens[b];
+  if (len < 0 || len > a.Lmax) {
+    if (threadIdx.x == 0 && split == 0 && hkv == 0) record_error(a.err, SBD_DEVERR_CACHE_LEN);
+    len = len < 0 ? 0 : a.Lmax;
+  }
+  const int n_cache_tiles = (len + kTileKeys - 1) / kTileKeys;
+  const int n_tiles = n_cache_tiles + 1;
+  const int t_begin = (int)((long long)split * n_tiles / a.splits);
+  const int t_end = (int)((long long)(split + 1) * n_tiles / a.splits);
+  const int n = t_end - t_begin;                  // 64-key tiles of this split
+  const int nt = (n + kTriTiles - 1) / kTriTiles; // triples (the last may be short)
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_sh;
+
+  if (warp == 0) {
+    // ------------------------------------------------ K producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap_k);
+      if (t_end == n_tiles) tma_prefetch_desc(&tmap_kb);
+      int issued = 0;
+      for (int t = 0; t < nt; ++t) {
+        const int slot = t % kWideKSlots;
+        if (!mbar_wait(&k_empty[slot], ((t / kWideKSlots) & 1) ^ 1, a.err)) break;
+        const int j0 = kTriTiles * t, ntl = min(kTriTiles, n - j0);
+        mbar_arrive_expect_tx(&k_full[slot], ntl * kSub * kKVSub);
+        for (int e = 0; e < ntl; ++e) {
+          const int j = j0 + e, tg = t_begin + j;
+          for (int h = 0; h < kSub; ++h) {
+            uint8_t* dst = smem_raw + (k_chunk(j, h) - smem_u32(smem_raw));
+            if (tg < n_cache_tiles)
+              tma_load_4d(dst, &tmap_k, &k_full[slot], 64 * h, hkv, tg * kTileKeys, b);
+            else   // the block keys; rows k..63 lie outside the block tensor: zeros
+              tma_load_4d(dst, &tmap_kb, &k_full[slot], 64 * h, hkv, 0, b);
+          }
+        }
+        issued = t + 1;
+      }
+      // copies still in flight land before the CTA exits (on every path the
+      // consumer would have waited for them; this matters only after a
+      // bounded wait gave up)
+      for (int t = issued - kWideKSlots > 0 ? issued - kWideKSlots : 0; t < issued; ++t)
+        mbar_wait(&k_full[t % kWideKSlots], (t / kWideKSlots) & 1, a.err);
+    }
+  } else if (warp == 2) {
+    // ------------------------------------------------ V producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap_v);
+      if (t_end == n_tiles) tma_prefetch_desc(&tmap_vb);
+    }
+    int issued = 0;
+    for (int j = 0; j < n; ++j) {
+      const int slot = j % kVSlots, tg = t_begin + j;
+      const bool freed = mbar_wait(&v_empty[slot], ((j / kVSlots) & 1) ^ 1, a.err);
+      if (!__all_sync(0xffffffffu, freed)) break;
+      issued = j + 1;
+      if (tg < n_cache_tiles) {
+        const int valid = min(kTileKeys, len - tg * kTileKeys);
+        const bool tail = valid < kTileKeys;
+        uint64_t* bar = tail ? &tail_bar : &v_full[slot];
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar, kSub * kKVSub);
+          for (int h = 0; h < kSub; ++h)
+            tma_load_4d(smem_raw + (v_chunk(j, h) - smem_u32(smem_raw)), &tmap_v, bar, 64 * h, hkv,
+                        tg * kTileKeys, b);
+        }
+        if (tail) {
+          // value rows past the length may hold anything (NaN): zero them so
+          // that zero probabilities stay zero
+          mbar_wait(&tail_bar, 0, a.err);
+          for (int c = lane; c < (kTileKeys - valid) * kSub * 8; c += 32) {
+            const int row = valid + c / (kSub * 8), h = (c / 8) % kSub, cc = c % 8;
+            st_shared_v4(swz(v_chunk(j, h), row, cc), make_uint4(0, 0, 0, 0));
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&v_full[slot]);
+        }
+      } else {
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&v_full[slot], kSub * kKVSub);
+          for (int h = 0; h < kSub; ++h)
+            tma_load_4d(smem_raw + (v_chunk(j, h) - smem_u32(smem_raw)), &tmap_vb, &v_full[slot],
+                        64 * h, hkv, 0, b);
+        }
+        if (a.kc_app) {
+          // first iteration of a block: the causal rows' keys and values also
+          // enter the cache at len .. len + n_causal - 1 (see attn_tc_kernel)
+          if (len + a.n_causal <= a.Lmax) {
+            constexpr int kCpr = kSub * 8;
+            constexpr int kBatch = 8;
+            const int n_app = a.n_causal * kCpr;
+            for (int c0 = 0; c0 < n_app; c0 += 32 * kBatch) {
+              uint4 kv[kBatch], vv[kBatch];
 #pragma unroll
-        for (int s2 = 0; s2 < 16; ++s2) {
-          if (s2 < S) {
-            const uint32_t src = mapa_shared(cpart_s + 4u * (r * kCStride + kPer * lane), s2);
-            if constexpr (kPer == 4) {
-              const float4 x = ld_cluster_v4(src);
-              v[s2][0] = x.x; v[s2][1] = x.y; v[s2][2] = x.z; v[s2][3] = x.w;
-            } else {
-              const float2 x = ld_cluster_v2(src);
-              v[s2][0] = x.x; v[s2][1] = x.y;
+              for (int e = 0; e < kBatch; ++e) {
+                const int c = c0 + e * 32 + lane;
+                if (c < n_app) {
+                  const size_t off = (((size_t)b * a.k + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
+                  kv[e] = *reinterpret_cast<const uint4*>(a.kb + off);
+                  vv[e] = *reinterpret_cast<const uint4*>(a.vb + off);
+                }
+              }
+#pragma unroll
+              for (int e = 0; e < kBatch; ++e) {
+                const int c = c0 + e * 32 + lane;
+                if (c < n_app) {
+                  const size_t dst =
+                      (((size_t)b * a.Lmax + len + c / kCpr) * a.Hkv + hkv) * D + (c % kCpr) * 8;
+                  *reinterpret_cast<uint4*>(a.kc_app + dst) = kv[e];
+                  *reinterpret_cast<uint4*>(a.vc_app + dst) = vv[e];
+                }
+              }
             }
+          } else if (lane == 0) {
+            record_error(a.err, SBD_DEVERR_CACHE_LEN);
           }
-        }
-        float acc[kPer];
-#pragma unroll
-        for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
-#pragma unroll
-        for (int s2 = 0; s2 < 16; ++s2) {
-          const float ws = __shfl_sync(0xffffffffu, w, s2);    // 0 past S
-          if (s2 < S && ws > 0.f) {
-#pragma unroll
-            for (int c = 0; c < kPer; ++c) acc[c] = fmaf(ws, v[s2][c], acc[c]);
-          }
-        }
-        const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-        __nv_bfloat16* dst =
-            a.out + (((size_t)b * a.k + r / a.G) * a.Hq + hkv * a.G + r % a.G) * D + kPer * lane;
-        if constexpr (kPer == 4) {
-          uint2 o2;
-          o2.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-          o2.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-          *reinterpret_cast<uint2*>(dst) = o2;
-        } else {
-          *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
         }
       }
     }
-    cluster_sync_all();
+    if (lane == 0)
+      for (int j = issued - kVSlots > 0 ? issued - kVSlots : 0; j < issued; ++j)
+        mbar_wait(&v_full[j % kVSlots], (j / kVSlots) & 1, a.err);
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0 && n > 0) {
+      const uint32_t id_o = idesc_bf16(kRows, D, true);
+      bool ok = mbar_wait(&q_ready, 0, a.err);
+      tc_fence_after();
+      auto issue_s = [&](int t) -> bool {
+        const int slot = t % kWideKSlots;
+        if (!mbar_wait(&k_full[slot], (t / kWideKSlots) & 1, a.err)) return false;
+        tc_fence_after();
+        const int ntl = min(kTriTiles, n - kTriTiles * t);
+        const uint32_t kb = k_chunk(kTriTiles * t, 0);
+        const uint32_t id_s = idesc_bf16(kRows, ntl * kTileKeys, false);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t ad = sw128_desc(q_s + (kk / 4) * kQBytes + (kk % 4) * 32, 16, 1024);
+          const uint64_t bd = sw128_desc(kb + (kk / 4) * kTriSub + (kk % 4) * 32, 16, 1024);
+          tc_mma(tmem, ad, bd, id_s, kk > 0);
+        }
+        tc_commit(&s_full);
+        tc_commit(&k_empty[slot]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int t = 0; t < nt && ok; ++t) {
+        // the next scores as soon as the softmax warps hold S_t in registers
+        if (t + 1 < nt) {
+          if (!mbar_wait(&s_free, t & 1, a.err)) break;
+          if (!issue_s(t + 1)) break;
+        }
+        if (!mbar_wait(&p_full[t & 1], (t >> 1) & 1, a.err)) break;
+        tc_fence_after();
+        const int j0 = kTriTiles * t, ntl = min(kTriTiles, n - j0);
+        for (int e = 0; e < ntl && ok; ++e) {
+          const int j = j0 + e;
+          if (!mbar_wait(&v_full[j % kVSlots], (j / kVSlots) & 1, a.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t vb = v_chunk(j, 0);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t bd = sw128_desc(vb + kk * 16 * 128, kKVSub, 1024);
+            tc_mma_ts(tmem + kOCol, tmem + kPCol + (t & 1) * kPStride + (4 * e + kk) * 8, bd, id_o,
+                      (t > 0 || e > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&v_empty[j % kVSlots]);
+        }
+        if (ok) tc_commit(&pv_done[t & 1]);
+      }
+    }
+  } else {
+    // ------------------------------------------------ softmax warps
+    const int sw = warp - 3;                     // 0..7
+    const int quad = warp & 3;                   // TMEM lanes 32*quad .. +31
+    const int sub = sw >> 2;                     // 0 or 1 within the quadrant
+    const int row = quad * 32 + lane;            // packed row = TMEM lane
+    const int cbase = kCW * sub;                 // this warp's columns of a triple
+    const int bar_id = 1 + quad;                 // the two warps of a quadrant
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    auto sw_of = [](int q_, int s_) { return 4 * s_ + ((q_ - 3) & 3); };
+    // Q row -> shared (swizzled, K-major); each sub-warp copies half a row;
+    // padding rows are zero.
+    {
+      const __nv_bfloat16* qrow =
+          row < a.M ? a.q + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
+                    : nullptr;
+#pragma unroll
+      for (int c = sub * (D / 16); c < (sub + 1) * (D / 16); ++c) {
+        const uint4 v = qrow ? *reinterpret_cast<const uint4*>(qrow + c * 8) : make_uint4(0, 0, 0, 0);
+        st_shared_v4(swz(q_s + (c / 8) * kQBytes, row, c % 8), v);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&q_ready);
+    }
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int t = 0; t < nt; ++t) {
+      // valid keys of the two tiles this warp's 96 columns fall in (sub 0:
+      // tile 0 and the first half of tile 1; sub 1: the second half of tile
+      // 1 and tile 2), for this row
+      auto valid_of = [&](int e) {
+        const int j = kTriTiles * t + e, tg = t_begin + j;
+        if (j >= n) return 0;
+        if (tg < n_cache_tiles) return min(kTileKeys, len - tg * kTileKeys);
+        return row / a.G < a.n_causal ? row / a.G + 1 : a.k;
+      };
+      const int valid_a = valid_of(sub), valid_b = valid_of(sub + 1);
+      const int off0 = cbase & (kTileKeys - 1);    // key of column 0 within its tile
+      if (ok && !mbar_wait(&s_full, t & 1, a.err)) ok = false;
+      ok = __all_sync(0xffffffffu, ok);
+      // the warp's 96 scores of this row, as raw fp32 bits
+      uint32_t sr[kCW / 16][16];
+      float mloc = -INFINITY;
+      if (ok) {
+        tc_fence_after();
+        const uint32_t sa = tmem + lane_addr + (uint32_t)cbase;
+#pragma unroll
+        for (int h = 0; h < kCW / 16; ++h) tc_ld16(sa + 16 * h, sr[h]);
+        tc_wait_ld();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free);
+        // column c is key off0 + c of the first tile while that is < 64, then
+        // key c - (64 - off0) of the second
+#pragma unroll
+        for (int c = 0; c < kCW; ++c) {
+          const bool first = c < kTileKeys - off0;
+          const int key = first ? off0 + c : c - (kTileKeys - off0);
+          if (key >= (first ? valid_a : valid_b)) sr[c / 16][c % 16] = __float_as_uint(-INFINITY);
+        }
+        float mx[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx[e] = __uint_as_float(sr[0][e]);
+#pragma unroll
+        for (int c = 8; c < kCW; c += 8)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], __uint_as_float(sr[c / 16][c % 16 + e]));
+        mloc = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      }
+      red_max[((t & 1) * kSoftWarps + sw) * 32 + lane] = bf16_bits_round_up(mloc);
+      asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(64) : "memory");
+      if (!ok) continue;
+      float mraw = -INFINITY;
+#pragma unroll
+      for (int s2 = 0; s2 < 2; ++s2)
+        mraw = fmaxf(mraw, bf16_bits_to_float(red_max[((t & 1) * kSoftWarps + sw_of(quad, s2)) * 32 + lane]));
+      const float mt = mraw * a.scale_log2;
+      const bool rescale = m_ref != -INFINITY && mt > m_ref + kRescaleThreshold;
+      const bool warp_rescale = __any_sync(0xffffffffu, rescale);
+      // P buffer t mod 2 is written after PV_{t-2}, O rescaled after PV_{t-1}
+      const int wait_t = warp_rescale ? t - 1 : t - 2;
+      bool waited = wait_t < 0 || mbar_wait(&pv_done[wait_t & 1], (wait_t >> 1) & 1, a.err);
+      if (!__all_sync(0xffffffffu, waited)) {
+        ok = false;
+        continue;
+      }
+      tc_fence_after();
+      const float alpha = rescale ? exp2f(m_ref - mt) : 1.f;
+      if (m_ref == -INFINITY) {
+        m_ref = mt;
+      } else if (rescale) {
+        l *= alpha;
+        m_ref = mt;
+      }
+      if (warp_rescale) {
+#pragma unroll
+        for (int c = sub * (D / 32); c < (sub + 1) * (D / 32); ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tc_st16(tmem + lane_addr + kOCol + c * 16, r);
+        }
+      }
+      // P = 2^(scale * s - m_ref) as bf16 pairs into tensor memory: this
+      // warp's 96 keys are P columns cbase / 2 .. + 47
+      {
+        const float nm = -m_ref;
+        float psum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int h = 0; h < kCW / 32; ++h) {
+          uint32_t r[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int c = 32 * h + 2 * e;
+            const float p0 = exp2f(fmaf(__uint_as_float(sr[c / 16][c % 16]), a.scale_log2, nm));
+            const float p1 = exp2f(fmaf(__uint_as_float(sr[(c + 1) / 16][(c + 1) % 16]), a.scale_log2, nm));
+            psum[(2 * e) & 7] += p0;
+            psum[(2 * e + 1) & 7] += p1;
+            r[e] = pack_bf16(p0, p1);
+          }
+          tc_st16(tmem + lane_addr + kPCol + (t & 1) * kPStride + cbase / 2 + 16 * h, r);
+        }
+        l += ((psum[0] + psum[1]) + (psum[2] + psum[3])) + ((psum[4] + psum[5]) + (psum[6] + psum[7]));
+      }
+      tc_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[t & 1]);
+    }
+    grid_dependents_launch();
+    // ------------------------------------------------ epilogue
+    asm volatile("bar.sync 5, %0;" ::"n"(kSoftWarps * 32) : "memory");
+    red_l[sw * 32 + lane] = l;
+    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(64) : "memory");
+    const float lsum = red_l[sw_of(quad, 0) * 32 + lane] + red_l[sw_of(quad, 1) * 32 + lane];
+    const bool mine = row < a.M;
+    const int c_lo = sub * (D / 32), c_hi = (sub + 1) * (D / 32);
+    bool final_ok = ok && nt > 0 && mbar_wait(&pv_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, a.err);
+    final_ok = __all_sync(0xffffffffu, final_ok);
+    constexpr int kCStride = D + 4;
+    float* cpart = reinterpret_cast<float*>(smem_raw + (k_s - smem_u32(smem_raw)));
+    float* clse = cpart + kRows * kCStride;
+    if (final_ok) {
+      tc_fence_after();
+      const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+      if (a.splits == 1) {
+        __nv_bfloat16* dst =
+            mine ? a.out + (((size_t)b * a.k + row / a.G) * a.Hq + hkv * a.G + row % a.G) * D
+                 : nullptr;
+#pragma unroll
+        for (int c = c_lo; c < c_hi; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+          if (mine) {
+            uint4 w0, w1;
+            w0.x = pack_bf16(__uint_as_float(r[0]) * inv, __uint_as_float(r[1]) * inv);
+            w0.y = pack_bf16(__uint_as_float(r[2]) * inv, __uint_as_float(r[3]) * inv);
+            w0.z = pack_bf16(__uint_as_float(r[4]) * inv, __uint_as_float(r[5]) * inv);
+            w0.w = pack_bf16(__uint_as_float(r[6]) * inv, __uint_as_float(r[7]) * inv);
+            w1.x = pack_bf16(__uint_as_float(r[8]) * inv, __uint_as_float(r[9]) * inv);
+            w1.y = pack_bf16(__uint_as_float(r[10]) * inv, __uint_as_float(r[11]) * inv);
+            w1.z = pack_bf16(__uint_as_float(r[12]) * inv, __uint_as_float(r[13]) * inv);
+            w1.w = pack_bf16(__uint_as_float(r[14]) * inv, __uint_as_float(r[15]) * inv);
+            *reinterpret_cast<uint4*>(dst + c * 16) = w0;
+            *reinterpret_cast<uint4*>(dst + c * 16 + 8) = w1;
+          }
+        }
+      } else {
+        const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
+        float* dst = mine ? (a.cluster ? cpart + row * kCStride : a.part_o + prow * D) : nullptr;
+#pragma unroll
+        for (int c = c_lo; c < c_hi; ++c) {
+          uint32_t r[16];
+          tc_ld16(tmem + lane_addr + kOCol + c * 16, r);
+          tc_wait_ld();
+          if (mine) {
+#pragma unroll
+            for (int e = 0; e < 16; e += 4)
+              *reinterpret_cast<float4*>(dst + c * 16 + e) =
+                  make_float4(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv,
+                              __uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
+          }
+        }
+        if (mine && sub == 0) {
+          const float lse = lsum > 0.f ? m_ref + log2f(lsum) : -INFINITY;
+          if (a.cluster) clse[row] = lse; else a.part_lse[prow] = lse;
+        }
+      }
+    } else if (n == 0 && a.splits > 1 && mine) {
+      const size_t prow = (((size_t)b * a.Hkv + hkv) * a.splits + split) * a.M + row;
+      float* dst = a.cluster ? cpart + row * kCStride : a.part_o + prow * D;
+      for (int d = c_lo * 16; d < c_hi * 16; ++d) dst[d] = 0.f;
+      if (sub == 0) {
+        if (a.cluster) clse[row] = -INFINITY; else a.part_lse[prow] = -INFINITY;
+      }
+    }
   }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tc_dealloc(tmem, kTmemCols);
+  }
+  if (a.cluster) cluster_merge<D>(a, b, hkv, k_s, warp - 3, lane);
 }
 
 }  // namespace
@@ -862,13 +1377,27 @@ size_t attn_tc_smem_bytes(int D) {
          (size_t)pairs * 2 * sub * kPairKeys * 128;
 }
 
-// The kernel instance for head dimension D and M packed rows (copies of
-// every row in the 128 MMA rows: 2 up to 64 rows, else 1).
-static const void* attn_tc_fn(int D, int M) {
-  const bool two = M <= kRows / 2;
-  if (D == 128)
-    return two ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<128, 1>;
-  return two ? (const void*)attn_tc_kernel<64, 2> : (const void*)attn_tc_kernel<64, 1>;
+static size_t attn_wide_smem_bytes(int D) {
+  const int sub = D / 64;
+  const int v_slots = D == 128 ? wide_v_slots<128>() : wide_v_slots<64>();
+  return 1024 + (size_t)sub * kRows * 128 + (size_t)kWideKSlots * sub * kTriKeys * 128 +
+         (size_t)v_slots * sub * kTileKeys * 128;
+}
+
+// The kernel for head dimension D and M packed rows: up to 64 rows
+// attn_tc_kernel with every row copied into both lane halves, above that
+// attn_wide_kernel.
+struct TcKernel {
+  const void* fn;
+  int threads;
+  size_t smem;
+};
+static TcKernel attn_tc_kernel_for(int D, int M) {
+  if (M <= kRows / 2)
+    return TcKernel{D == 128 ? (const void*)attn_tc_kernel<128, 2> : (const void*)attn_tc_kernel<64, 2>,
+                    kThreads, attn_tc_smem_bytes(D)};
+  return TcKernel{D == 128 ? (const void*)attn_wide_kernel<128> : (const void*)attn_wide_kernel<64>,
+                  kWideThreads, attn_wide_smem_bytes(D)};
 }
 
 bool attn_tc_cluster_ok(const AttnPlan& p, int splits) {
@@ -889,7 +1418,8 @@ bool attn_tc_cluster_ok(const AttnPlan& p, int splits) {
     cudaGetLastError();
     return false;
   }
-  const void* fn = attn_tc_fn(p.D, p.M);
+  const TcKernel kern = attn_tc_kernel_for(p.D, p.M);
+  const void* fn = kern.fn;
   int clusters = -1;
   {
     std::lock_guard<std::mutex> lock(mu);
@@ -898,8 +1428,8 @@ bool attn_tc_cluster_ok(const AttnPlan& p, int splits) {
         clusters = cache[i].clusters;
   }
   if (clusters < 0) {
-    clusters = max_active_clusters(fn, dim3(splits, p.Hkv, p.B), dim3(kThreads),
-                                   attn_tc_smem_bytes(p.D), splits);
+    clusters = max_active_clusters(fn, dim3(splits, p.Hkv, p.B), dim3(kern.threads), kern.smem,
+                                   splits);
     std::lock_guard<std::mutex> lock(mu);
     if (n_cache < 32) cache[n_cache++] = Entry{dev, fn, splits, clusters};
   }
@@ -933,8 +1463,9 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   a.vc_app = (__nv_bfloat16*)vc_app;
   a.scale_log2 = p.scale_log2;
   a.cluster = p.cluster ? 1 : 0;
-  const size_t smem = attn_tc_smem_bytes(p.D);
-  const void* fn = attn_tc_fn(p.D, p.M);
+  const TcKernel kern = attn_tc_kernel_for(p.D, p.M);
+  const size_t smem = kern.smem;
+  const void* fn = kern.fn;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
   // The block keys/values [B, k, Hkv, D] as 4-D tensors (D, Hkv, k, B), read
@@ -955,7 +1486,7 @@ sbd_status attn_tc_launch(const AttnPlan& p, const CUtensorMap& tk, const CUtens
   }
   CUtensorMap k_map = tk, v_map = tv;
   void* args[] = {(void*)&k_map, (void*)&v_map, (void*)&kb_map, (void*)&vb_map, (void*)&a};
-  return launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(kThreads), smem, st, args,
+  return launch_pdl(fn, dim3(p.splits, p.Hkv, p.B), dim3(kern.threads), smem, st, args,
                     "attn_tc_kernel launch", p.cluster ? p.splits : 1);
 }
 

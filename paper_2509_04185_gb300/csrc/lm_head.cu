@@ -366,11 +366,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int ring_bytes = a.ring_bytes + head_scratch_bytes(a.rows_alloc) - ep_bytes;
   uint8_t* ring = gbase + ep_bytes;
   const uint32_t rbase = sbase + ep_bytes;
-  StatsRef wstats[4];
-  for (int w = 0; w < 4; ++w) {
-    wstats[w].msTb = reinterpret_cast<float4*>(ep) + w * n_eff;
-    wstats[w].idx = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * sizeof(float4)) + w * n_eff;
-  }
+  // Statistics of TMEM lane quadrant w (computed, not indexed from an array:
+  // a per-thread array of the four would live in local memory).
+  auto wstats = [&](int w) -> StatsRef {
+    StatsRef r;
+    r.msTb = reinterpret_cast<float4*>(ep) + w * n_eff;
+    r.idx = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * sizeof(float4)) + w * n_eff;
+    return r;
+  };
   int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * (sizeof(float4) + 4));
   // Ring shape from the actual row count: a stage holds `boxes` 64-column
   // boxes of W (16 KB each) and of the n_eff hidden rows.  Above two boxes,
@@ -410,7 +413,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     const int te = threadIdx.x - 64;
     for (int i = te; i < n_eff; i += kEpiThreads) {
       rmap[i] = (!kLinear && i < R) ? a.row_map[i] : 0;
-      for (int w = 0; w < 4; ++w) store_stats(wstats[w], i, rowstats_empty());
+      for (int w = 0; w < 4; ++w) store_stats(wstats(w), i, rowstats_empty());
     }
   }
   tc_fence_before();
@@ -503,6 +506,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     } else {
       // ------------------------------------------------ epilogue warps
       const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
+      const StatsRef my_stats = wstats(quad);
       const int sub = (warp - 2) / 4;          // chunks sub, sub + n_sub, ... of 16 columns
       const bool noisy = !kLinear && a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
@@ -602,7 +606,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
             const RowStats st = chunk16_stats(z, g, valid, a.tau, v0, lane);
             const int col = c0 + ((lane >> 1) & 15);
             if ((lane & 1) == 0 && col < R)
-              store_stats(wstats[quad], col, rowstats_merge(load_stats(wstats[quad], col), st));
+              store_stats(my_stats, col, rowstats_merge(load_stats(my_stats, col), st));
           }
         }
         tc_fence_before();
@@ -613,8 +617,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const int te = threadIdx.x - 64;
       if constexpr (!kLinear) {
         for (int col = te; col < R; col += kEpiThreads) {
-          RowStats s = load_stats(wstats[0], col);
-          for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats[w], col));
+          RowStats s = load_stats(wstats(0), col);
+          for (int w = 1; w < 4; ++w) s = rowstats_merge(s, load_stats(wstats(w), col));
           const size_t o = (size_t)blockIdx.x * a.rows_alloc + col;
           a.part_msTb[o] = make_float4(s.m, s.S, s.T, s.best);
           a.part_idx[o] = s.idx;
