@@ -1208,12 +1208,15 @@ attn_wide_kernel(const __grid_constant__ CUtensorMap tmap_k,
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_free);
         // column c is key off0 + c of the first tile while that is < 64, then
-        // key c - (64 - off0) of the second
+        // key c - (64 - off0) of the second; masked keys exist only in the
+        // last cache tile, the block tile and past the split's last tile
+        if (valid_a < kTileKeys || valid_b < kTileKeys) {
 #pragma unroll
-        for (int c = 0; c < kCW; ++c) {
-          const bool first = c < kTileKeys - off0;
-          const int key = first ? off0 + c : c - (kTileKeys - off0);
-          if (key >= (first ? valid_a : valid_b)) sr[c / 16][c % 16] = __float_as_uint(-INFINITY);
+          for (int c = 0; c < kCW; ++c) {
+            const bool first = c < kTileKeys - off0;
+            const int key = first ? off0 + c : c - (kTileKeys - off0);
+            if (key >= (first ? valid_a : valid_b)) sr[c / 16][c % 16] = __float_as_uint(-INFINITY);
+          }
         }
         float mx[8];
 #pragma unroll
