@@ -333,10 +333,10 @@ attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
       float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
       for (int n = 0; n < kNT; ++n) {
-        s[n][0] = exp2f(s[n][0] - mu0);
-        s[n][1] = exp2f(s[n][1] - mu0);
-        s[n][2] = exp2f(s[n][2] - mu1);
-        s[n][3] = exp2f(s[n][3] - mu1);
+        s[n][0] = ex2_ftz(s[n][0] - mu0);
+        s[n][1] = ex2_ftz(s[n][1] - mu0);
+        s[n][2] = ex2_ftz(s[n][2] - mu1);
+        s[n][3] = ex2_ftz(s[n][3] - mu1);
         ps0 += s[n][0] + s[n][1];
         ps1 += s[n][2] + s[n][3];
       }

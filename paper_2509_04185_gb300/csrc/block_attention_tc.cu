@@ -728,7 +728,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           float p[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            p[e] = exp2f(fmaf(s[c * 8 + e], a.scale_log2, nm));
+            p[e] = ex2_ftz(fmaf(s[c * 8 + e], a.scale_log2, nm));
             psum[e] += p[e];
           }
           st_shared_v4(swz(pb, lane_t, coff / 8 + c),
@@ -1275,8 +1275,8 @@ attn_wide_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
             const int c = 32 * h + 2 * e;
-            const float p0 = exp2f(fmaf(__uint_as_float(sr[c / 16][c % 16]), a.scale_log2, nm));
-            const float p1 = exp2f(fmaf(__uint_as_float(sr[(c + 1) / 16][(c + 1) % 16]), a.scale_log2, nm));
+            const float p0 = ex2_ftz(fmaf(__uint_as_float(sr[c / 16][c % 16]), a.scale_log2, nm));
+            const float p1 = ex2_ftz(fmaf(__uint_as_float(sr[(c + 1) / 16][(c + 1) % 16]), a.scale_log2, nm));
             psum[(2 * e) & 7] += p0;
             psum[(2 * e + 1) & 7] += p1;
             r[e] = pack_bf16(p0, p1);

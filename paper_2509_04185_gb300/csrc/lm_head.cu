@@ -210,7 +210,7 @@ __device__ __forceinline__ RowStats chunk16_stats(const float (&z)[16], const fl
     const float m = __shfl_sync(0xffffffffu, ms[0], 2 * j);
     const float best = __shfl_sync(0xffffffffu, mb[0], 2 * j);
     const float d = s[j] - m;                  // <= 0 on valid lanes
-    e[j] = valid ? exp2f(d) : 0.f;
+    e[j] = valid ? ex2_ftz(d) : 0.f;
     t[j] = valid ? e[j] * d : 0.f;
     const unsigned hits = __ballot_sync(0xffffffffu, valid && sc[j] == best);
     if (my_col == j) my_hits = hits;

@@ -264,6 +264,14 @@ __device__ __forceinline__ void grid_dependents_launch() {
 }
 
 // ---- warp-level helpers
+// 2^x by the SFU's ex2.approx.ftz instruction (PTX ISA: max relative error
+// about 2^-22; results below 2^-126 flush to zero).  For probabilities that
+// are rounded to bf16 or summed in fp32 right after.
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
