@@ -802,6 +802,11 @@ def run_sweep(args):
     head_bytes_first = V * H * e + B * k * H * e + (B * k * V * 4 if args.noise == "buffer" else 0)
     ms_per_step = total_ms / n_steps
     attn_gbs = attn_bytes / (attn_ms * 1e-3) / 1e9
+    # DRAM bytes of one layer's attention launch from the committed capture
+    # (while the kernel source is unchanged), times the layers of a step
+    per_launch = profiled_traffic(args.workload, os.path.join(
+        ROOT, "paper_2509_04185_gb300", "csrc", "block_attention_tc.cu"))
+    sweep_traffic = int(per_launch * NL) if per_launch else None
     line = {
         "metric": METRIC, "value": round(job_us_per_step(total_ms, n_steps, world), 3), "unit": UNIT,
         "n_gpus": world, "steps": n_steps, "warmup": args.warmup,
@@ -820,11 +825,11 @@ def run_sweep(args):
         "per_call_us": {"attention_32_layers": round(attn_ms * 1000, 3),
                         "head": round(head_ms * 1000, 3), "eb_select": round(eb_ms * 1000, 3)},
         "roofline": {
-            "kernel": "block attention, 32 layers (attn_tc_kernel, or attn_bf16_kernel at "
-                      "16 packed rows or fewer, + split combine when split)",
+            "kernel": "block attention, 32 layers (attn_tc_kernel up to 64 packed rows, "
+                      "attn_wide_kernel above, attn_bf16_kernel at 16 or fewer)",
             "bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"],
             "peak_source": peak_src, "unit": "GB/s", "frac": round(attn_gbs / peaks["hbm_gbs"], 4),
-            "traffic": None, "algorithmic_bytes": int(attn_bytes)},
+            "traffic": sweep_traffic, "algorithmic_bytes": int(attn_bytes)},
         "head_first_step_bytes": int(head_bytes_first),
         "host_wall_s": round(wall, 3),
         "clocks": clocks, "e2e": None, "cpu_baseline": None,
