@@ -62,7 +62,7 @@ BF16 = gen.get_workload("llama8b_k16")
 
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("G,k", [(4, 1), (4, 4), (1, 16), (4, 8), (3, 7), (2, 9), (4, 12), (4, 16),
-                                 (2, 40 // 2), (4, 32), (8, 16)])
+                                 (2, 40 // 2), (4, 32), (8, 16), (3, 25), (5, 20), (2, 32)])
 def test_bf16_shapes(sbd, D, G, k):
     Hkv = 2
     w = gen.shrink(BF16, batch=2, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv, head_dim=D,
@@ -81,6 +81,15 @@ def test_bf16_ragged_edges(sbd):
     w = gen.shrink(BF16, batch=5, block_k=8, n_q_heads=8, n_kv_heads=2, cache_len=(0, 129))
     _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=2)
     _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=1)
+
+
+@pytest.mark.parametrize("k,splits", [(8, 5), (8, 16), (32, 1), (32, 2), (32, 7)])
+def test_bf16_ragged_edges_every_kernel(sbd, k, splits):
+    """Lengths 0, 1, 64, 65 and 129 through both tcgen05 kernels (32 and 128
+    packed rows), with splits merged in a cluster (2, 5, 7, 16 splits, some
+    of them empty) or unsplit."""
+    w = gen.shrink(BF16, batch=5, block_k=k, n_q_heads=8, n_kv_heads=2, cache_len=(0, 129))
+    _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=splits)
 
 
 def test_bf16_scale_override(sbd):
