@@ -29,6 +29,8 @@
 // linear_reduce_kernel sums).
 #include <math.h>
 
+#include <mutex>
+
 #include "philox.cuh"
 #include "sbd_internal.cuh"
 
@@ -132,6 +134,103 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          | (1u << 7)                // A format: bf16
          | (1u << 10)               // B format: bf16
          | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ---- the CTA-pair (2-SM) forms.  Two CTAs of a cluster share one MMA of
+// M = 256: each holds 128 rows of A and half of B's N rows (rank 0 the first
+// half) at the same shared-memory offsets, and each gets its 128 rows of D
+// in its own tensor memory.  Every tcgen05 instruction of a pair kernel uses
+// cta_group::2; allocation and release are performed by one warp of each
+// CTA together.
+__device__ __forceinline__ void tc_alloc_pair(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// Issued by one thread of the pair's rank-0 CTA.
+__device__ __forceinline__ void tc_mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc,
+                                                 uint64_t b_desc, uint32_t idesc,
+                                                 uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// One arrival on the mbarrier at this offset in every CTA of `cta_mask`
+// once the pair's tcgen05 ops issued so far by this thread have completed.
+__device__ __forceinline__ void tc_commit_pair(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(cta_mask)
+      : "memory");
+}
+// TMA load into this CTA's shared memory whose completion is counted on an
+// mbarrier of either CTA of the pair (bar: shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar,
+                                                 int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile"
+      ".mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair_hint(void* dst, const CUtensorMap* map,
+                                                      uint32_t bar, int c0, int c1,
+                                                      uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile"
+      ".mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void pair_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t pair_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The shared::cluster address of this CTA's shared location `p` in the
+// pair's rank-0 CTA.
+__device__ __forceinline__ uint32_t at_rank0(const void* p) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(r) : "r"(smem_u32(p)));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar)
+               : "memory");
+}
+// mbar_wait for a barrier that CTAs of the cluster arrive on.
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, int* err) {
+  const uint64_t t0 = globaltimer();
+  for (uint32_t n = 0;; ++n) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if ((n & 63u) == 63u && globaltimer() - t0 > kWaitLimitNs) {
+      record_error(err, SBD_DEVERR_TIMEOUT);
+      return false;
+    }
+  }
 }
 
 // ------------------------------------------------------------ epilogue math
@@ -634,6 +733,529 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   }
 }
 
+// ------------------------------------------------------------ bf16 tcgen05, CTA pairs
+// head_pair_kernel: the LM head on CTA pairs (clusters of 2) running 2-SM
+// MMAs of M = 256.  A unit of work is a pair tile of 256 vocabulary rows
+// (128 W rows in each CTA).  Both CTAs' copies complete on rank 0's full
+// barriers; rank 0's thread issues the MMAs and commits them to the barriers
+// of both CTAs; the epilogue warps of rank 1 release an accumulator on rank
+// 0's barrier.  Two layouts, chosen from the live row count R:
+//  - Rows mode (R > kPairVocabLanesMax): the hidden rows are the A side
+//    (TMEM lane = hidden row, 128 per CTA) and W the B side (N = 256), so
+//    that each CTA's accumulator holds its rows' logits over all 256 ids of
+//    the tile.  Each epilogue thread owns one row and folds its logits into
+//    running statistics in registers, with no exchange between lanes; the
+//    two warps of a lane quadrant take alternate 16-column chunks and merge
+//    at the end.  Above 256 live rows there are two row groups; the pairs
+//    take one group each, and the two pairs of a tile run at the same time
+//    (W's lines come from L2 for the second).
+//  - Vocabulary mode (R <= kPairVocabLanesMax): as in head_tc_kernel, W is
+//    the A side (TMEM lane = vocabulary row) and the live rows the B side
+//    (N = R padded to 32, half of them in each CTA), with the column
+//    reductions over lanes.  The MMA's work then grows with R instead of
+//    being fixed at 256 rows.
+// Measured on GB300: a 2-SM MMA of N = 256 takes ~65 ns, against ~95 ns for
+// the same work per SM as a 1-SM MMA, and each SM reads half of the hidden
+// rows from L2.  The column reductions over lanes took ~28 us per 256 x 128
+// logits, which bounds the vocabulary layout from ~200 rows; below that the
+// rows layout's fixed 256-row MMAs cost power (the kernel ran at ~1750 MHz
+// and ~950 W at 60 live rows, against 2070 MHz and ~450 W for
+// head_tc_kernel) and lost to it.
+constexpr int kPairRows = 128;                 // hidden rows of one CTA per unit (M / 2)
+constexpr int kPairVocabLanesMax = 192;        // live rows up to which the vocabulary layout runs
+
+// One 16-column chunk of a row's logits z (vocabulary ids v0 .. v0 + 15, valid
+// below V) and Gumbel noise g folded into the running statistics.
+__device__ __forceinline__ void fold_chunk16(RowStats& st, const float (&z)[16],
+                                             const float (&g)[16], float tau, int v0, int V) {
+  float y[16];
+  float mc = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    y[j] = v0 + j < V ? z[j] * kLog2e : -INFINITY;
+    mc = fmaxf(mc, y[j]);
+  }
+  if (mc == -INFINITY) return;                  // no valid id in this chunk
+  const float m_new = fmaxf(st.m, mc);
+  float s_add = 0.f, t_add = 0.f;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    // invalid ids: 2^-1000 flushes to 0, and 0 * -1000 adds nothing to T
+    const float d = v0 + j < V ? y[j] - m_new : -1000.f;
+    const float e = ex2_ftz(d);
+    s_add += e;
+    t_add = fmaf(e, d, t_add);
+  }
+  if (st.S > 0.f) {
+    // rescale the old sums to the new maximum: T' = 2^dm (T + dm S)
+    const float dm = st.m - m_new;
+    const float alpha = ex2_ftz(dm);
+    st.T = fmaf(alpha, fmaf(dm, st.S, st.T), t_add);
+    st.S = fmaf(alpha, st.S, s_add);
+  } else {
+    st.T = t_add;
+    st.S = s_add;
+  }
+  st.m = m_new;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    // ids ascend within the chunk: a strict > keeps the lowest id on ties
+    const float sc = fmaf(tau, g[j], z[j]);
+    if (v0 + j < V && sc > st.best) {
+      st.best = sc;
+      st.idx = v0 + j;
+    }
+  }
+}
+
+template <bool kPhilox>
+__global__ void __launch_bounds__(kHeadThreads, 1)
+head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                 const __grid_constant__ CUtensorMap tmap_h,
+                 const __grid_constant__ CUtensorMap tmap_h64,
+                 const __grid_constant__ CUtensorMap tmap_h128, const HeadArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t tmem_full[2];
+  __shared__ __align__(8) uint64_t tmem_empty[2];
+  __shared__ __align__(8) uint64_t drain_bar;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ float4 half_msTb[kPairRows];   // the second warp of each quadrant's row statistics
+  __shared__ int half_idx[kPairRows];
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (sbase - smem_u32(smem_raw));
+  const int rank = (int)pair_rank();
+  const int pair = (int)(blockIdx.x >> 1), n_pairs = (int)(gridDim.x >> 1);
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_h);
+  }
+  // Everything below reads what the compaction kernel wrote.
+  grid_dependency_wait();
+  const int R = *a.n_rows;
+  // The layout: hidden rows on the lanes above kPairVocabLanesMax live rows,
+  // vocabulary rows on the lanes up to it.
+  const bool rows_mode = R > kPairVocabLanesMax;
+  // Row groups of 2 x 128 rows (rows mode); each pair takes one group and
+  // every per_group-th tile from its first one.
+  const int n_groups = R > 2 * kPairRows ? 2 : 1;
+  const int per_group = n_pairs / n_groups;
+  const int grp = pair % n_groups;
+  const bool working = R > 0 && pair < per_group * n_groups;
+  const int t_first = pair / n_groups;
+  // this CTA's hidden rows row0 .. row0 + 127 (live below R), and the peer's
+  const int row0 = grp * 2 * kPairRows + rank * kPairRows;
+  auto live_rows = [&](int r0) { return R - r0 < 0 ? 0 : (R - r0 > kPairRows ? kPairRows : R - r0); };
+  const int live = live_rows(row0);
+  const int live16 = (live + 15) / 16 * 16;                       // rows loaded
+  const int peer16 = (live_rows(grp * 2 * kPairRows + (1 - rank) * kPairRows) + 15) / 16 * 16;
+  // Ring: a stage holds `boxes` 64-column boxes of the hidden rows, then as
+  // many of W (128 rows).  A hidden box takes the rows rank 0 of the group
+  // loads (the larger share; the same layout in both CTAs): the MMA reads
+  // 128 rows from its start, and the rows past the live ones come from the
+  // next box or from W in the same stage, landed and only feeding the
+  // accumulator lanes of rows that are not live.  So the ring holds as much
+  // W as the live rows leave room for; as many boxes as still leave 3 stages.
+  //
+  // Vocabulary mode: the live rows padded to G (a multiple of 32), each CTA
+  // loading G / 2 of them as its half of the B side; a stage holds `boxes`
+  // boxes of W, then as many of the hidden rows.  The epilogue's running
+  // statistics (per lane quadrant and row) and the row map sit in shared
+  // memory before the ring.
+  const int G = ((R > 0 ? R : 1) + 31) / 32 * 32;
+  const int n_eff = R <= 16 ? 16 : (R + 15) / 16 * 16;
+  const int ep_bytes = rows_mode ? 0 : head_scratch_bytes(n_eff);
+  uint8_t* ep = gbase;
+  uint8_t* ring = gbase + ep_bytes;
+  const uint32_t rbase = sbase + (uint32_t)ep_bytes;
+  const int ring_bytes = a.ring_bytes - ep_bytes;
+  const int h_box = rows_mode ? ((live_rows(grp * 2 * kPairRows) + 15) / 16 * 16) * kBK * 2
+                              : (G / 2) * kBK * 2;
+  int boxes = kMaxBoxes;
+  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || ring_bytes / (boxes * (kABytes + h_box)) < 3))
+    boxes >>= 1;
+  const int stage_bytes = boxes * (kABytes + h_box);
+  int stages = ring_bytes / stage_bytes;
+  if (stages > kMaxStages) stages = kMaxStages;
+  const int num_kb = a.H / (kBK * boxes);                          // stages per unit
+  // offsets in a stage of W box x and hidden box x; the hidden rows loaded
+  const int w_off0 = rows_mode ? boxes * h_box : 0;
+  const int h_off0 = rows_mode ? 0 : boxes * kABytes;
+  const int h_first = rows_mode ? row0 : rank * (G / 2);
+  const int h_count = rows_mode ? live16 : G / 2;
+  // bytes landing per stage on rank 0's barrier: W and hidden rows of both CTAs
+  const uint32_t tx_pair = rows_mode
+      ? (uint32_t)boxes * (2u * kABytes + (uint32_t)(live16 + peer16) * 128u)
+      : 2u * (uint32_t)stage_bytes;
+  // vocabulary mode: statistics of TMEM lane quadrant w, and the row map
+  auto wstats = [&](int w) -> StatsRef {
+    StatsRef r;
+    r.msTb = reinterpret_cast<float4*>(ep) + w * n_eff;
+    r.idx = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * sizeof(float4)) + w * n_eff;
+    return r;
+  };
+  int* rmap = reinterpret_cast<int*>(ep + (size_t)4 * n_eff * (sizeof(float4) + 4));
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tmem_full[i], 1);
+      mbar_init(&tmem_empty[i], 2 * kEpiWarps);   // every epilogue warp of both CTAs
+    }
+    mbar_init(&drain_bar, 1);
+    fence_mbar_init();
+  }
+  if (!rows_mode && warp >= 2) {
+    for (int i = threadIdx.x - 64; i < n_eff; i += kEpiThreads) {
+      rmap[i] = i < R ? a.row_map[i] : 0;
+      for (int w = 0; w < 4; ++w) store_stats(wstats(w), i, rowstats_empty());
+    }
+  }
+  // Both CTAs run and their barriers are initialised before either one
+  // signals the other's; the pair then allocates its tensor memory.
+  pair_sync();
+  if (warp == 1) tc_alloc_pair(&tmem_base_sh, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_base_sh;
+
+  if (working) {
+    if (warp == 0) {
+      // ------------------------------------------------ TMA producer
+      if (lane == 0) {
+        // W is read once: evict-first, except where two row groups share it
+        const bool w_hint = n_groups == 1;
+        const uint64_t policy = l2_policy_evict_first();
+        int it = 0;
+        bool ok = true;
+        for (int t = t_first; ok && t < a.n_tiles; t += per_group) {
+          const int w_row = (2 * t + rank) * kBM;
+          for (int kb = 0; kb < num_kb; ++kb, ++it) {
+            const int s = it % stages;
+            const uint32_t ph = (it / stages) & 1;
+            if (!mbar_wait(&empty_bar[s], ph ^ 1, a.err)) {
+              ok = false;
+              break;
+            }
+            uint8_t* st = ring + (size_t)s * stage_bytes;
+            if (rank == 0) mbar_arrive_expect_tx(&full_bar[s], tx_pair);
+            const uint32_t fb = at_rank0(&full_bar[s]);
+            for (int x = 0; x < boxes; ++x) {
+              const int col = (kb * boxes + x) * kBK;
+              uint8_t* wb = st + w_off0 + x * kABytes;
+              if (w_hint) tma_load_2d_pair_hint(wb, &tmap_w, fb, col, w_row, policy);
+              else tma_load_2d_pair(wb, &tmap_w, fb, col, w_row);
+              // the hidden rows in the tallest boxes that fit (from L2)
+              uint8_t* hb = st + h_off0 + x * h_box;
+              int r0 = 0;
+              if (a.h_big >= 128)
+                for (; r0 + 128 <= h_count; r0 += 128)
+                  tma_load_2d_pair(hb + r0 * 128, &tmap_h128, fb, col, h_first + r0);
+              if (a.h_big >= 64)
+                for (; r0 + 64 <= h_count; r0 += 64)
+                  tma_load_2d_pair(hb + r0 * 128, &tmap_h64, fb, col, h_first + r0);
+              for (; r0 < h_count; r0 += 16)
+                tma_load_2d_pair(hb + r0 * 128, &tmap_h, fb, col, h_first + r0);
+            }
+          }
+        }
+        // Copies still in flight must land before the CTA exits.  Rank 1
+        // cannot wait on rank 0's full barriers: it waits until the MMAs
+        // released its last stages, which they do only after they arrived.
+        bool landed = true;
+        for (int q = it - stages > 0 ? it - stages : 0; landed && q < it; ++q)
+          landed = rank == 0 ? mbar_wait(&full_bar[q % stages], (q / stages) & 1, a.err)
+                             : mbar_wait(&empty_bar[q % stages], (q / stages) & 1, a.err);
+      }
+    } else if (warp == 1) {
+      // ------------------------------------------------ MMA issuer (rank 0)
+      if (lane == 0 && rank == 0) {
+        // rows mode: A = hidden rows, B = W (N = 256 vocabulary ids);
+        // vocabulary mode: A = W, B = hidden rows (N = G)
+        const uint32_t idesc = idesc_bf16_f32(2 * kPairRows, rows_mode ? 2 * kBM : G);
+        int it = 0, local = 0;
+        bool ok = true;
+        for (int t = t_first; ok && t < a.n_tiles; t += per_group, ++local) {
+          const int acc = local & 1;
+          const uint32_t use = (uint32_t)(local >> 1);
+          // both CTAs' epilogue warps release the accumulator here
+          if (!mbar_wait_cluster(&tmem_empty[acc], (use & 1) ^ 1, a.err)) break;
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + (uint32_t)acc * 256u;
+          for (int kb = 0; kb < num_kb; ++kb, ++it) {
+            const int s = it % stages;
+            const uint32_t ph = (it / stages) & 1;
+            if (!mbar_wait(&full_bar[s], ph, a.err)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = rbase + (uint32_t)(s * stage_bytes);
+            for (int x = 0; x < boxes; ++x) {
+              const uint32_t w_s = st + (uint32_t)(w_off0 + x * kABytes);
+              const uint32_t h_s = st + (uint32_t)(h_off0 + x * h_box);
+              const uint64_t adesc = sw128_kmajor_desc(rows_mode ? h_s : w_s);
+              const uint64_t bdesc = sw128_kmajor_desc(rows_mode ? w_s : h_s);
+#pragma unroll
+              for (int kk = 0; kk < kBK / 16; ++kk)
+                tc_mma_bf16_pair(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc,
+                                 (kb != 0 || x != 0 || kk != 0) ? 1u : 0u);
+            }
+            tc_commit_pair(&empty_bar[s], 0x3);
+          }
+          if (ok) tc_commit_pair(&tmem_full[acc], 0x3);
+        }
+        // the MMAs read both CTAs' shared memory: none may be in flight when
+        // the pair leaves (this matters after a time-out only)
+        tc_commit_pair(&drain_bar, 0x1);
+        mbar_wait(&drain_bar, 0, a.err);
+      }
+    } else if (rows_mode) {
+      // ------------------------------------------------ epilogue warps, rows mode
+      const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31
+      const int sub = (warp - 2) >> 2;         // 16-column chunks sub, sub + 2, ... of a unit
+      const int h = row0 + quad * 32 + lane;   // this thread's hidden row
+      const bool row_live = h < R;
+      const bool warp_live = __any_sync(0xffffffffu, row_live);
+      const int n = row_live ? a.row_map[h] : 0;
+      const bool noisy = a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
+      const float* grow = noisy && !kPhilox ? a.gumbel + (size_t)n * a.V : nullptr;
+      const bool vec4 = ((reinterpret_cast<uintptr_t>(a.gumbel) | (uintptr_t)a.V * 4u) & 15u) == 0;
+      const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+      constexpr int kChunks = 2 * kBM / 16 / 2;   // chunks of one warp per unit
+      auto load_noise = [&](int v0, float (&g)[16]) {
+        if (!(noisy && row_live)) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) g[j] = 0.f;
+        } else if constexpr (kPhilox) {
+          // one call gives the words of ids 4q .. 4q + 3 (v0 is a multiple of 16)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const uint4 x = sbd_philox::philox4x32_10(
+                make_uint4(((uint32_t)v0 >> 2) + (uint32_t)i, (uint32_t)n, a.off_lo, a.off_hi),
+                a.seed_lo, a.seed_hi);
+#pragma unroll
+            for (int w = 0; w < 4; ++w) g[4 * i + w] = sbd_philox::gumbel_of_word(sbd_philox::word_of(x, w));
+          }
+        } else if (vec4) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float4 q4 = v0 + 4 * i < a.V ? __ldg(reinterpret_cast<const float4*>(grow + v0) + i)
+                                               : make_float4(0.f, 0.f, 0.f, 0.f);
+            g[4 * i] = q4.x;
+            g[4 * i + 1] = q4.y;
+            g[4 * i + 2] = q4.z;
+            g[4 * i + 3] = q4.w;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) g[j] = v0 + j < a.V ? __ldg(grow + v0 + j) : 0.f;
+        }
+      };
+      RowStats st = rowstats_empty();
+      int local = 0;
+      for (int t = t_first; t < a.n_tiles; t += per_group, ++local) {
+        const int acc = local & 1;
+        const uint32_t use = (uint32_t)(local >> 1);
+        const int vt = t * 2 * kBM;                     // first vocabulary id of the tile
+        const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)acc * 256u;
+        // noise of the first kGAhead chunks is read while the MMAs run
+        float gq[kGAhead][16];
+        if constexpr (!kPhilox) {
+#pragma unroll
+          for (int d = 0; d < kGAhead; ++d) load_noise(vt + 16 * (sub + 2 * d), gq[d]);
+        }
+        // the tcgen05.ld below is warp-collective: the warp goes on as a whole
+        if (!__all_sync(0xffffffffu, mbar_wait(&tmem_full[acc], use & 1, a.err))) break;
+        tc_fence_after();
+        if (warp_live) {
+#pragma unroll 1
+          for (int c = 0; c < kChunks; ++c) {
+            const int col = 16 * (sub + 2 * c);
+            float g[16];
+            if constexpr (!kPhilox) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) g[j] = gq[0][j];
+#pragma unroll
+              for (int d = 0; d + 1 < kGAhead; ++d)
+#pragma unroll
+                for (int j = 0; j < 16; ++j) gq[d][j] = gq[d + 1][j];
+              if (c + kGAhead < kChunks) load_noise(vt + col + 32 * kGAhead, gq[kGAhead - 1]);
+            } else {
+              load_noise(vt + col, g);
+            }
+            uint32_t r[16];
+            tc_ld_32x32b_x16(t_acc + (uint32_t)col, r);
+            tc_wait_ld();
+            if (row_live) {
+              float z[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
+              fold_chunk16(st, z, g, a.tau, vt + col, a.V);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 1) mbar_arrive_cluster(at_rank0(&tmem_empty[acc]));
+          else mbar_arrive(&tmem_empty[acc]);
+        }
+      }
+      // the two warps of a quadrant merge their halves of each row
+      const int slot = quad * 32 + lane;
+      if (sub == 1) {
+        half_msTb[slot] = make_float4(st.m, st.S, st.T, st.best);
+        half_idx[slot] = st.idx;
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+      if (sub == 0 && row_live) {
+        RowStats o;
+        o.m = half_msTb[slot].x;
+        o.S = half_msTb[slot].y;
+        o.T = half_msTb[slot].z;
+        o.best = half_msTb[slot].w;
+        o.idx = half_idx[slot];
+        st = rowstats_merge(st, o);
+        const size_t off = (size_t)blockIdx.x * a.rows_alloc + h;
+        a.part_msTb[off] = make_float4(st.m, st.S, st.T, st.best);
+        a.part_idx[off] = st.idx;
+      }
+    } else {
+      // ------------------------------------------------ epilogue warps, vocabulary mode
+      // As in head_tc_kernel: thread = vocabulary row (TMEM lane), chunks of
+      // 16 hidden-row columns reduced over the warp (chunk16_stats) and
+      // merged into the quadrant's statistics in shared memory.
+      const int quad = warp & 3;
+      const StatsRef my_stats = wstats(quad);
+      const int sub = (warp - 2) >> 2;          // chunks sub, sub + 2, ... of 16 columns
+      const bool noisy = a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
+      const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+      constexpr int kStride = 32;
+      const int c_first = 16 * sub;
+      int local = 0;
+      for (int t = t_first; t < a.n_tiles; t += per_group, ++local) {
+        const int acc = local & 1;
+        const uint32_t use = (uint32_t)(local >> 1);
+        const int v0 = (2 * t + rank) * kBM + quad * 32;
+        const int v = v0 + lane;
+        const bool valid = v < a.V;
+        const uint32_t t_acc = tmem_base + lane_addr + (uint32_t)acc * 256u;
+        // Gumbel noise of the first kGAhead chunks is loaded while the MMAs
+        // run; each chunk's reduction then loads the chunk kGAhead further on.
+        float gq[kGAhead][16];
+        if constexpr (!kPhilox) {
+#pragma unroll
+          for (int d = 0; d < kGAhead; ++d)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int cn = c_first + d * kStride + j;
+              gq[d][j] = (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            }
+        }
+        // the tcgen05.ld below is warp-collective: the warp goes on as a whole
+        if (!__all_sync(0xffffffffu, mbar_wait(&tmem_full[acc], use & 1, a.err))) break;
+        tc_fence_after();
+        for (int c0 = c_first; c0 < R; c0 += kStride) {
+          float g[16];
+          if constexpr (!kPhilox) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) g[j] = gq[0][j];
+#pragma unroll
+            for (int d = 0; d + 1 < kGAhead; ++d)
+#pragma unroll
+              for (int j = 0; j < 16; ++j) gq[d][j] = gq[d + 1][j];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int cn = c0 + kGAhead * kStride + j;
+              gq[kGAhead - 1][j] =
+                  (noisy && valid && cn < R) ? __ldg(a.gumbel + (size_t)rmap[cn] * a.V + v) : 0.f;
+            }
+          } else if (noisy) {
+            // lanes 4q .. 4q + 3 share one Philox counter per row: each lane
+            // computes the calls of 4 of the chunk's 16 rows, and a 4 x 4
+            // transpose inside the group gives every lane word v mod 4 of all 16
+            const uint32_t vq = (uint32_t)v >> 2;
+            const int i4 = lane & 3;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int rr = c0 + 4 * q + i4;
+              const uint32_t n = rr < R ? (uint32_t)rmap[rr] : 0u;
+              const uint4 x = sbd_philox::philox4x32_10(make_uint4(vq, n, a.off_lo, a.off_hi),
+                                                        a.seed_lo, a.seed_hi);
+              uint32_t b[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+              for (int d = 0; d < 4; ++d) {
+                const uint32_t send = sbd_philox::word_of(x, i4 ^ d);
+                const uint32_t recv = d == 0 ? send : __shfl_xor_sync(0xffffffffu, send, d);
+#pragma unroll
+                for (int jj = 0; jj < 4; ++jj) b[jj] = (jj == (i4 ^ d)) ? recv : b[jj];
+              }
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj) g[4 * q + jj] = sbd_philox::gumbel_of_word(b[jj]);
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) g[j] = 0.f;
+          }
+          uint32_t r[16];
+          tc_ld_32x32b_x16(t_acc + (uint32_t)c0, r);
+          tc_wait_ld();
+          float z[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
+          const RowStats cs = chunk16_stats(z, g, valid, a.tau, v0, lane);
+          const int col = c0 + ((lane >> 1) & 15);
+          if ((lane & 1) == 0 && col < R)
+            store_stats(my_stats, col, rowstats_merge(load_stats(my_stats, col), cs));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 1) mbar_arrive_cluster(at_rank0(&tmem_empty[acc]));
+          else mbar_arrive(&tmem_empty[acc]);
+        }
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+      for (int col = threadIdx.x - 64; col < R; col += kEpiThreads) {
+        RowStats m4 = load_stats(wstats(0), col);
+        for (int w = 1; w < 4; ++w) m4 = rowstats_merge(m4, load_stats(wstats(w), col));
+        const size_t off = (size_t)blockIdx.x * a.rows_alloc + col;
+        a.part_msTb[off] = make_float4(m4.m, m4.S, m4.T, m4.best);
+        a.part_idx[off] = m4.idx;
+      }
+    }
+  }
+  // Partials of the live rows this CTA does not own (rows mode, or no work):
+  // empty statistics (the combine merges every CTA's partial of every row).
+  if (warp >= 2 && (rows_mode || !working)) {
+    const RowStats e = rowstats_empty();
+    for (int r = threadIdx.x - 64; r < R; r += kEpiThreads) {
+      if (working && r >= row0 && r < row0 + kPairRows) continue;
+      const size_t off = (size_t)blockIdx.x * a.rows_alloc + r;
+      a.part_msTb[off] = make_float4(e.m, e.S, e.T, e.best);
+      a.part_idx[off] = e.idx;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  // neither CTA releases its tensor memory or leaves while the other may
+  // still signal its barriers or read its shared memory
+  pair_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tc_dealloc_pair(tmem_base, 512);
+  }
+  pair_sync();
+}
+
 // ------------------------------------------------------------ fp32 SIMT
 // One CTA per 128 vocab rows; z by sequential fp32 FMAs over H; the same
 // column statistics as the tensor-core epilogue.
@@ -808,6 +1430,43 @@ size_t head_smem_bytes(int rows_alloc) {
   return 1024 + (size_t)head_scratch_bytes(rows_alloc) + head_ring_bytes(rows_alloc);
 }
 
+// The LM head runs on CTA pairs (head_pair_kernel) from this many allocated
+// rows; its shared memory is the ring alone.
+constexpr int kPairMinRows = 64;
+// its ring: what is left of the 227 KB of a CTA next to its static shared
+// memory (barriers and 2.5 KB of row statistics) and the 1 KB alignment
+constexpr int kPairRingBytes = 222 * 1024;
+constexpr size_t kPairSmemBytes = 1024 + kPairRingBytes;
+
+// How many clusters of two CTAs of `fn` the current device holds at once
+// (0: none).  Kept per (device, kernel): the call is on every launch's host
+// path.
+int head_pair_slots(const void* fn) {
+  struct Entry {
+    int dev;
+    const void* fn;
+    int clusters;
+  };
+  static std::mutex mu;
+  static Entry cache[16];
+  static int n_cache = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < n_cache; ++i)
+      if (cache[i].dev == dev && cache[i].fn == fn) return cache[i].clusters;
+  }
+  const int clusters =
+      sbd::max_active_clusters(fn, dim3(2), dim3(kHeadThreads), kPairSmemBytes, 2);
+  std::lock_guard<std::mutex> lock(mu);
+  if (n_cache < 16) cache[n_cache++] = Entry{dev, fn, clusters};
+  return clusters;
+}
+
 // y = the sum over K ranges of the fp32 partials of sbd_linear, in bf16.
 __global__ void __launch_bounds__(256)
 linear_reduce_kernel(const float* __restrict__ part, int ksplit, long long tn,
@@ -887,6 +1546,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
   }
   cudaError_t e;
   int* err = device_error_word();
+  int n_parts = p.n_ctas;   // CTAs that write per-row partials
   if (p.bf16) {
     CUtensorMap tw, th, th64, th128;
     {
@@ -939,22 +1599,47 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     a.ksplit = 1;
     a.part_y = nullptr;
     a.h_big = p.rows_alloc >= 128 ? 128 : (p.rows_alloc >= 64 ? 64 : 16);
-    a.ring_bytes = head_ring_bytes(p.rows_alloc);
-    // tensor memory for two accumulators of the allocated width (one of it
-    // above 256 rows); the kernel picks the buffer count from the live rows
-    const int n_acc_alloc = 2 * p.rows_alloc <= 512 ? 2 : 1;
-    uint32_t cols = 32;
-    while (cols < (uint32_t)(n_acc_alloc * p.rows_alloc)) cols <<= 1;
-    a.tmem_cols = cols;
     a.tau = tau;
-    const size_t smem = head_smem_bytes(p.rows_alloc);
-    const void* fn = philox ? (const void*)head_tc_kernel<true, false>
-                            : (const void*)head_tc_kernel<false, false>;
+    // CTA pairs from kPairMinRows allocated rows: as many as the device holds
+    // at once, the pair tiles need and the workspace has partials for
+    // (p.n_ctas), an even number when there may be two row groups.
+    const void* fn_pair = philox ? (const void*)head_pair_kernel<true>
+                                 : (const void*)head_pair_kernel<false>;
+    const int pair_tiles = (p.V + 2 * kBM - 1) / (2 * kBM);
+    const int n_groups_max = p.rows_alloc > 2 * kPairRows ? 2 : 1;
+    int n_pairs = 0;
+    if (p.rows_alloc >= kPairMinRows && p.n_ctas >= 2) {
+      n_pairs = head_pair_slots(fn_pair);
+      if (n_pairs > pair_tiles * n_groups_max) n_pairs = pair_tiles * n_groups_max;
+      if (n_pairs > p.n_ctas / 2) n_pairs = p.n_ctas / 2;
+      if (n_groups_max == 2) n_pairs &= ~1;
+    }
+    const void* fn;
+    size_t smem;
+    if (n_pairs > 0) {
+      fn = fn_pair;
+      smem = kPairSmemBytes;
+      a.ring_bytes = kPairRingBytes;
+      a.n_tiles = pair_tiles;
+      a.tmem_cols = 512;
+      n_parts = 2 * n_pairs;
+    } else {
+      fn = philox ? (const void*)head_tc_kernel<true, false> : (const void*)head_tc_kernel<false, false>;
+      smem = head_smem_bytes(p.rows_alloc);
+      a.ring_bytes = head_ring_bytes(p.rows_alloc);
+      // tensor memory for two accumulators of the allocated width (one of it
+      // above 256 rows); the kernel picks the buffer count from the live rows
+      const int n_acc_alloc = 2 * p.rows_alloc <= 512 ? 2 : 1;
+      uint32_t cols = 32;
+      while (cols < (uint32_t)(n_acc_alloc * p.rows_alloc)) cols <<= 1;
+      a.tmem_cols = cols;
+    }
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel)");
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(LM head kernel)");
     void* args[] = {(void*)&tw, (void*)&th, (void*)&th64, (void*)&th128, (void*)&a};
-    s = launch_pdl(fn, dim3(p.n_ctas), dim3(kHeadThreads), smem, st, args,
-                   "head_tc_kernel launch");
+    s = launch_pdl(fn, dim3(n_parts), dim3(kHeadThreads), smem, st, args,
+                   n_pairs > 0 ? "head_pair_kernel launch" : "head_tc_kernel launch",
+                   n_pairs > 0 ? 2 : 1);
     if (s != SBD_OK) return s;
   } else {
     const float* hc = (const float*)W.hidden_c;
@@ -979,7 +1664,7 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
   {
     const float4* pm = W.part_msTb;
     const int32_t* pi = W.part_idx;
-    int np = p.n_ctas, ra = p.rows_alloc;
+    int np = n_parts, ra = p.rows_alloc;
     const int32_t* rm = W.row_map;
     const int32_t* nr = W.n_rows;
     void* args[] = {(void*)&pm, (void*)&pi, (void*)&np,      (void*)&ra,   (void*)&rm,

@@ -74,11 +74,14 @@ def test_bf16_shapes(sbd, B, k, V, H, tau):
     assert compare_head(d, "bf16", tau, ent, tok, with_noise=tau != 0.0) <= 1
 
 
-@pytest.mark.parametrize("R", [64, 80, 128, 144, 192, 208, 256, 320])
+@pytest.mark.parametrize("R", [1, 17, 64, 80, 128, 144, 192, 193, 208, 255, 256, 257, 320, 400, 511,
+                               512])
 def test_bf16_hidden_box_decomposition(sbd, R):
-    """Exactly R masked rows out of 512: the live rows are loaded in boxes of
-    128, 64 and 16 rows (144 = 128 + 16, 208 = 128 + 64 + 16; above 256 the
-    MMA N splits); every row must come out right."""
+    """Exactly R masked rows out of 512 (the CTA-pair kernel): the live rows
+    are loaded in boxes of 128, 64 and 16 rows (144 = 128 + 16,
+    208 = 128 + 64 + 16); up to 192 rows the vocabulary-lane layout, from
+    193 the row-lane layout, from 257 with two row groups; every row must
+    come out right."""
     w = gen.shrink(gen.get_workload("llama8b_k16"), batch=16, block_k=32, vocab=1100, hidden=192,
                    cache_len=16)
     d = step_inputs(w, seed=R)
@@ -130,12 +133,14 @@ def test_full_size_configs(sbd, name):
     np.testing.assert_array_equal(ent, ent0)                  # entropy independent of tau
 
 
-def test_sweep_first_step_512_rows(sbd):
-    """The first step of a k = 32 block of the 32-layer sweep: batch 16,
-    all 512 block positions masked, hidden 4096, vocab 128256 (the
-    compute-bound, single-accumulator path of the kernel), at tau = 1 and
-    tau = 0, against one evaluation of the oracle's logits."""
-    w = gen.sweep_workload(32)
+@pytest.mark.parametrize("k", [16, 32])
+def test_sweep_first_step(sbd, k):
+    """The first step of a k = 16 or k = 32 block of the 32-layer sweep:
+    batch 16, all 256 or 512 block positions masked, hidden 4096, vocab
+    128256 (the compute-bound row-lane layout of the CTA-pair kernel, with
+    one or two row groups), at tau = 1 and tau = 0, against one evaluation
+    of the oracle's logits."""
+    w = gen.sweep_workload(k)
     B, k, V, H = w.batch, w.block_k, w.vocab, w.hidden
     d = {"w": cached_weight(V, H, "bf16", 0), "hidden": gen.hidden_states(w, 0, 0),
          "gumbel": gen.gumbel_noise(w, 0, 0), "masked": np.ones((B, k), dtype=np.uint8)}
@@ -144,7 +149,7 @@ def test_sweep_first_step_512_rows(sbd):
     np.testing.assert_array_equal(ent1, ent0)
     rent, rtok1, zs = oracle.head_entropy_sample(oracle.widen(d["hidden"], "bf16"), d["w"], "bf16",
                                                  d["masked"], d["gumbel"], 1.0)
-    assert len(zs) == 512
+    assert len(zs) == B * k
     assert np.abs(ent1 - rent).max() <= ENTROPY_TOL
     acc = H // 16
     exempt = 0
@@ -155,5 +160,5 @@ def test_sweep_first_step_512_rows(sbd):
                 gap = top2_gap(z, g, tau)
                 assert gap < token_tolerance(z, acc), (b, i, tau, tok[b, i], want, gap)
                 exempt += 1
-    print(f"token exemptions: {exempt} of 1024")
+    print(f"token exemptions: {exempt} of {2 * B * k}")
     assert exempt <= 2

@@ -32,12 +32,17 @@ def test_noise_tensor_matches_oracle(sbd, rows, V, seed, offset):
     assert np.abs(g - ref).max() < NOISE_TOL
 
 
-def _case(B, k, V, H, dtype, seed):
+def _case(B, k, V, H, dtype, seed, n_masked=None):
     w = gen.shrink(gen.get_workload("llama8b_k16"), batch=B, block_k=k, vocab=V, hidden=H,
                    dtype=dtype)
     rng = np.random.default_rng(seed)
-    masked = (rng.uniform(size=(B, k)) < 0.7).astype(np.uint8)
-    masked[0, -1] = 1
+    if n_masked is None:
+        masked = (rng.uniform(size=(B, k)) < 0.7).astype(np.uint8)
+        masked[0, -1] = 1
+    else:
+        masked = np.zeros(B * k, dtype=np.uint8)
+        masked[rng.choice(B * k, size=n_masked, replace=False)] = 1
+        masked = masked.reshape(B, k)
     return {"w": cached_weight(V, H, dtype, seed), "hidden": gen.hidden_states(w, seed, 0),
             "masked": masked}
 
@@ -48,8 +53,20 @@ def _case(B, k, V, H, dtype, seed):
                                            (1, 16, 128256, 4096, "bf16")])
 @pytest.mark.parametrize("tau", [1.0, 0.3])
 def test_head_with_philox_noise(sbd, B, k, V, H, dtype, tau):
+    _check_philox_head(sbd, _case(B, k, V, H, dtype, seed=B * 7 + k), B, k, V, H, dtype, tau)
+
+
+@pytest.mark.parametrize("R", [100, 200, 300])
+def test_head_with_philox_noise_row_counts(sbd, R):
+    """Exactly R of 512 rows masked: the CTA-pair kernel's vocabulary-lane
+    layout (R <= 192), its row-lane layout with one row group (193..256)
+    and with two (above 256)."""
+    B, k, V, H = 16, 32, 3001, 256
+    _check_philox_head(sbd, _case(B, k, V, H, "bf16", seed=R, n_masked=R), B, k, V, H, "bf16", 1.0)
+
+
+def _check_philox_head(sbd, d, B, k, V, H, dtype, tau):
     import torch
-    d = _case(B, k, V, H, dtype, seed=B * 7 + k)
     seed, offset = 1234567 + B, 99 + k
     hid = to_dev(d["hidden"], dtype)
     W = to_dev(d["w"], dtype)
