@@ -487,7 +487,7 @@ def run_ours(args):
         "attention_hbm_gbs": round(attn_gbs, 1),
         "tokens_committed_per_s": round(n_accepted / (ms_per_step * 1e-3) * world, 1),
         "roofline": {
-            "kernel": "LM head call (compact_rows + head_tc_kernel tcgen05 + head_combine)",
+            "kernel": "LM head call (compact_rows + head_tc_kernel or head_pair_kernel, tcgen05 + head_combine)",
             "bound": "hbm", "achieved": round(achieved, 1),
             "peak": peaks["hbm_gbs"], "peak_source": peak_src, "unit": "GB/s",
             "frac": round(achieved / peaks["hbm_gbs"], 4),
