@@ -208,10 +208,12 @@ sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t voc
  *                                   when the size is 0)
  *
  * y is the fp32 sum over in_features of the bf16 products, rounded to
- * bf16 (round to nearest even).  At up to 64 rows the in_features are cut
- * into ranges summed in fp32 by a second kernel through the workspace, so
- * that narrow layers still spread over all SMs.  All pointers 16-byte
- * aligned, caller-owned.  Asynchronous on `stream`.
+ * bf16 (round to nearest even).  When a layer has too few output tiles to
+ * fill the GPU, the in_features are cut into ranges whose fp32 partials go
+ * through the workspace and are summed by a second kernel (the split is
+ * chosen per call from the shape).  Above 192 rows the product runs on
+ * pairs of SMs (2-SM tensor-core MMAs).  All pointers 16-byte aligned,
+ * caller-owned.  Asynchronous on `stream`.
  * Supported: dtype bf16, 0 <= rows <= 512, in_features a positive multiple
  * of 64, out_features >= 1; SBD_ERR_UNSUPPORTED otherwise; a workspace
  * smaller than needed gives SBD_ERR_WORKSPACE.
@@ -221,8 +223,9 @@ typedef struct {
   sbd_dtype dtype;
 } sbd_linear_desc;
 
-/* Bytes for the largest split the call may choose (the same on every
- * device; 0 above 64 rows); 0 for an invalid descriptor. */
+/* Bytes for the largest split the call may choose: a function of the
+ * shape only, the same on every device (0 when no split is possible); 0
+ * for an invalid descriptor. */
 size_t sbd_linear_workspace_size(const sbd_linear_desc* desc);
 sbd_status sbd_linear(const sbd_linear_desc* desc, const void* x, const void* w, void* y,
                       void* workspace, size_t workspace_bytes, void* stream);

@@ -808,7 +808,17 @@ __device__ __forceinline__ void fold_chunk16(RowStats& st, const float (&z)[16],
   }
 }
 
-template <bool kPhilox>
+// kLinear: sbd_linear's product y = x W^T (all rows of x live, no noise),
+// always in the rows layout, the epilogue storing each row's outputs; with
+// a.ksplit > 1 each (pair tile, K range) is a unit and the epilogue stores
+// fp32 partials for linear_reduce_kernel.
+// Two values rounded to bf16 (nearest even), the first in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+template <bool kPhilox, bool kLinear>
 __global__ void __launch_bounds__(kHeadThreads, 1)
 head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
                  const __grid_constant__ CUtensorMap tmap_h,
@@ -823,6 +833,7 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   __shared__ uint32_t tmem_base_sh;
   __shared__ float4 half_msTb[kPairRows];   // the second warp of each quadrant's row statistics
   __shared__ int half_idx[kPairRows];
+  static_assert(!(kPhilox && kLinear), "the linear form has no noise");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
@@ -836,10 +847,10 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   }
   // Everything below reads what the compaction kernel wrote.
   grid_dependency_wait();
-  const int R = *a.n_rows;
+  const int R = kLinear ? a.linear_rows : *a.n_rows;
   // The layout: hidden rows on the lanes above kPairVocabLanesMax live rows,
   // vocabulary rows on the lanes up to it.
-  const bool rows_mode = R > kPairVocabLanesMax;
+  const bool rows_mode = kLinear || R > kPairVocabLanesMax;
   // Row groups of 2 x 128 rows (rows mode); each pair takes one group and
   // every per_group-th tile from its first one.
   const int n_groups = R > 2 * kPairRows ? 2 : 1;
@@ -847,6 +858,10 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int grp = pair % n_groups;
   const bool working = R > 0 && pair < per_group * n_groups;
   const int t_first = pair / n_groups;
+  // kLinear: K ranges per pair tile; a "tile" index below runs over
+  // (pair tile, K range) pairs
+  const int ksplit = kLinear ? a.ksplit : 1;
+  const int n_tk = a.n_tiles * ksplit;
   // this CTA's hidden rows row0 .. row0 + 127 (live below R), and the peer's
   const int row0 = grp * 2 * kPairRows + rank * kPairRows;
   auto live_rows = [&](int r0) { return R - r0 < 0 ? 0 : (R - r0 > kPairRows ? kPairRows : R - r0); };
@@ -876,12 +891,13 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int h_box = rows_mode ? ((live_rows(grp * 2 * kPairRows) + 15) / 16 * 16) * kBK * 2
                               : (G / 2) * kBK * 2;
   int boxes = kMaxBoxes;
-  while (boxes > 1 && ((a.H / kBK) % boxes != 0 || ring_bytes / (boxes * (kABytes + h_box)) < 3))
+  while (boxes > 1 &&
+         ((a.H / kBK) % (boxes * ksplit) != 0 || ring_bytes / (boxes * (kABytes + h_box)) < 3))
     boxes >>= 1;
   const int stage_bytes = boxes * (kABytes + h_box);
   int stages = ring_bytes / stage_bytes;
   if (stages > kMaxStages) stages = kMaxStages;
-  const int num_kb = a.H / (kBK * boxes);                          // stages per unit
+  const int num_kb = a.H / (kBK * boxes) / ksplit;                 // stages per unit
   // offsets in a stage of W box x and hidden box x; the hidden rows loaded
   const int w_off0 = rows_mode ? boxes * h_box : 0;
   const int h_off0 = rows_mode ? 0 : boxes * kABytes;
@@ -935,7 +951,8 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint64_t policy = l2_policy_evict_first();
         int it = 0;
         bool ok = true;
-        for (int t = t_first; ok && t < a.n_tiles; t += per_group) {
+        for (int tk = t_first; ok && tk < n_tk; tk += per_group) {
+          const int t = tk / ksplit, kb0 = (tk % ksplit) * num_kb;
           const int w_row = (2 * t + rank) * kBM;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
             const int s = it % stages;
@@ -948,7 +965,7 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
             if (rank == 0) mbar_arrive_expect_tx(&full_bar[s], tx_pair);
             const uint32_t fb = at_rank0(&full_bar[s]);
             for (int x = 0; x < boxes; ++x) {
-              const int col = (kb * boxes + x) * kBK;
+              const int col = ((kb0 + kb) * boxes + x) * kBK;
               uint8_t* wb = st + w_off0 + x * kABytes;
               if (w_hint) tma_load_2d_pair_hint(wb, &tmap_w, fb, col, w_row, policy);
               else tma_load_2d_pair(wb, &tmap_w, fb, col, w_row);
@@ -982,7 +999,7 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const uint32_t idesc = idesc_bf16_f32(2 * kPairRows, rows_mode ? 2 * kBM : G);
         int it = 0, local = 0;
         bool ok = true;
-        for (int t = t_first; ok && t < a.n_tiles; t += per_group, ++local) {
+        for (int tk = t_first; ok && tk < n_tk; tk += per_group, ++local) {
           const int acc = local & 1;
           const uint32_t use = (uint32_t)(local >> 1);
           // both CTAs' epilogue warps release the accumulator here
@@ -1024,9 +1041,12 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const int h = row0 + quad * 32 + lane;   // this thread's hidden row
       const bool row_live = h < R;
       const bool warp_live = __any_sync(0xffffffffu, row_live);
-      const int n = row_live ? a.row_map[h] : 0;
-      const bool noisy = a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
+      const int n = !kLinear && row_live ? a.row_map[h] : 0;
+      const bool noisy = !kLinear && a.tau != 0.f && (kPhilox || a.gumbel != nullptr);
       const float* grow = noisy && !kPhilox ? a.gumbel + (size_t)n * a.V : nullptr;
+      // kLinear: 16-byte stores of 8 outputs where the row stride allows
+      const bool y_vec = ((reinterpret_cast<uintptr_t>(a.y) | (uintptr_t)a.V * 2u) & 15u) == 0;
+      const bool p_vec = ((reinterpret_cast<uintptr_t>(a.part_y) | (uintptr_t)a.V * 4u) & 15u) == 0;
       const bool vec4 = ((reinterpret_cast<uintptr_t>(a.gumbel) | (uintptr_t)a.V * 4u) & 15u) == 0;
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       constexpr int kChunks = 2 * kBM / 16 / 2;   // chunks of one warp per unit
@@ -1061,7 +1081,8 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
       };
       RowStats st = rowstats_empty();
       int local = 0;
-      for (int t = t_first; t < a.n_tiles; t += per_group, ++local) {
+      for (int tk = t_first; tk < n_tk; tk += per_group, ++local) {
+        const int t = tk / ksplit, ks = tk % ksplit;
         const int acc = local & 1;
         const uint32_t use = (uint32_t)(local >> 1);
         const int vt = t * 2 * kBM;                     // first vocabulary id of the tile
@@ -1098,7 +1119,45 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
               float z[16];
 #pragma unroll
               for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(r[j]);
-              fold_chunk16(st, z, g, a.tau, vt + col, a.V);
+              if constexpr (kLinear) {
+                // y[h, vt + col + j], j < 16, below out_features (a.V), or
+                // with K ranges the fp32 partial of range ks
+                const int n0 = vt + col;
+                if (ksplit > 1) {
+                  float* pr = a.part_y + ((size_t)ks * R + h) * a.V + n0;
+                  if (p_vec && n0 + 16 <= a.V) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                      reinterpret_cast<float4*>(pr)[i] =
+                          make_float4(z[4 * i], z[4 * i + 1], z[4 * i + 2], z[4 * i + 3]);
+                  } else {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                      if (n0 + j < a.V) pr[j] = z[j];
+                  }
+                } else {
+                  __nv_bfloat16* yr = a.y + (size_t)h * a.V + n0;
+                  if (y_vec && n0 + 16 <= a.V) {
+                    uint4 q0, q1;
+                    q0.x = pack_bf16x2(z[0], z[1]);
+                    q0.y = pack_bf16x2(z[2], z[3]);
+                    q0.z = pack_bf16x2(z[4], z[5]);
+                    q0.w = pack_bf16x2(z[6], z[7]);
+                    q1.x = pack_bf16x2(z[8], z[9]);
+                    q1.y = pack_bf16x2(z[10], z[11]);
+                    q1.z = pack_bf16x2(z[12], z[13]);
+                    q1.w = pack_bf16x2(z[14], z[15]);
+                    reinterpret_cast<uint4*>(yr)[0] = q0;
+                    reinterpret_cast<uint4*>(yr)[1] = q1;
+                  } else {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                      if (n0 + j < a.V) yr[j] = __float2bfloat16_rn(z[j]);
+                  }
+                }
+              } else {
+                fold_chunk16(st, z, g, a.tau, vt + col, a.V);
+              }
             }
           }
         }
@@ -1111,6 +1170,7 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
       }
       // the two warps of a quadrant merge their halves of each row
       const int slot = quad * 32 + lane;
+      if constexpr (!kLinear) {
       if (sub == 1) {
         half_msTb[slot] = make_float4(st.m, st.S, st.T, st.best);
         half_idx[slot] = st.idx;
@@ -1128,7 +1188,8 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
         a.part_msTb[off] = make_float4(st.m, st.S, st.T, st.best);
         a.part_idx[off] = st.idx;
       }
-    } else {
+      }
+    } else if constexpr (!kLinear) {
       // ------------------------------------------------ epilogue warps, vocabulary mode
       // As in head_tc_kernel: thread = vocabulary row (TMEM lane), chunks of
       // 16 hidden-row columns reduced over the warp (chunk16_stats) and
@@ -1235,7 +1296,7 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   }
   // Partials of the live rows this CTA does not own (rows mode, or no work):
   // empty statistics (the combine merges every CTA's partial of every row).
-  if (warp >= 2 && (rows_mode || !working)) {
+  if (!kLinear && warp >= 2 && (rows_mode || !working)) {
     const RowStats e = rowstats_empty();
     for (int r = threadIdx.x - 64; r < R; r += kEpiThreads) {
       if (working && r >= row0 && r < row0 + kPairRows) continue;
@@ -1603,8 +1664,8 @@ sbd_status head_launch(const HeadPlan& p, const void* hidden, const void* w,
     // CTA pairs from kPairMinRows allocated rows: as many as the device holds
     // at once, the pair tiles need and the workspace has partials for
     // (p.n_ctas), an even number when there may be two row groups.
-    const void* fn_pair = philox ? (const void*)head_pair_kernel<true>
-                                 : (const void*)head_pair_kernel<false>;
+    const void* fn_pair = philox ? (const void*)head_pair_kernel<true, false>
+                                 : (const void*)head_pair_kernel<false, false>;
     const int pair_tiles = (p.V + 2 * kBM - 1) / (2 * kBM);
     const int n_groups_max = p.rows_alloc > 2 * kPairRows ? 2 : 1;
     int n_pairs = 0;
@@ -1719,6 +1780,34 @@ int linear_ksplit(int T, int K, int N) {
   return best;
 }
 
+// K ranges for the CTA-pair linear (rows layout): the same kind of time
+// model per pair of SMs.  A unit streams 128 W rows x K / ks per SM
+// (~45 GB/s per SM at the HBM peak) or runs K / (16 ks) 2-SM MMAs of
+// ~65 ns, whichever is longer; with ranges it also writes its rows' fp32
+// partials, and the sum over ranges reads them all back in a second launch.
+// At most linear_max_split (what the workspace holds).
+static int pair_linear_ksplit(int T, int K, int N, int n_pairs) {
+  const int max_ks = linear_max_split(T, K, N);
+  const int pair_tiles = (N + 2 * kBM - 1) / (2 * kBM);
+  const int n_groups = T > 2 * kPairRows ? 2 : 1;
+  const int per_group = n_pairs / n_groups > 0 ? n_pairs / n_groups : 1;
+  const double t_mem = 128.0 * K * 2 / 45e3, t_mma = K / 16.0 * 0.065;   // us
+  const double t_unit = t_mem > t_mma ? t_mem : t_mma;
+  const int rows_cta = (T < 2 * kPairRows ? T : 2 * kPairRows) / 2;
+  const double t_part = (double)rows_cta * 2 * kBM * 4 / 45e3;
+  int best = 1;
+  double best_cost = (double)((pair_tiles + per_group - 1) / per_group) * t_unit;
+  for (int ks = 2; ks <= max_ks; ks *= 2) {
+    const double waves = (double)((pair_tiles * ks + per_group - 1) / per_group);
+    const double cost = waves * (t_unit / ks + t_part) + (double)ks * T * N * 4 / 6e6 + 2.0;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = ks;
+    }
+  }
+  return best;
+}
+
 size_t linear_workspace_bytes(int T, int K, int N) {
   const int ks = linear_max_split(T, K, N);
   return ks > 1 ? (size_t)ks * T * N * sizeof(float) : 0;
@@ -1728,7 +1817,6 @@ sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void
                          cudaStream_t st) {
   if (T == 0 || N == 0) return SBD_OK;
   const int rows_alloc = T <= 16 ? 16 : ((T + 15) / 16) * 16;
-  const int ksplit = linear_ksplit(T, K, N);
   CUtensorMap tw, tx, tx64, tx128;
   sbd_status s;
   {
@@ -1769,26 +1857,58 @@ sbd_status linear_launch(int T, int K, int N, const void* x, const void* w, void
   a.rows_alloc = rows_alloc;
   a.n_tiles = (N + kBM - 1) / kBM;
   a.h_big = T >= 128 ? 128 : (T >= 64 ? 64 : 16);
-  a.ring_bytes = head_ring_bytes(rows_alloc);
-  const int n_acc_alloc = 2 * rows_alloc <= 512 ? 2 : 1;
-  uint32_t cols = 32;
-  while (cols < (uint32_t)(n_acc_alloc * rows_alloc)) cols <<= 1;
-  a.tmem_cols = cols;
   a.tau = 0.f;
   a.y = (__nv_bfloat16*)y;
   a.linear_rows = T;
-  a.ksplit = ksplit;
   a.part_y = (float*)ws;
-  const size_t smem = head_smem_bytes(rows_alloc);
-  const void* fn = (const void*)head_tc_kernel<false, true>;
+  // Above the pair kernel's vocabulary-lane limit: CTA pairs in the rows
+  // layout, as many as the device holds at once and the units need (an
+  // even number with two row groups), with their own choice of K ranges.
+  int ksplit = linear_ksplit(T, K, N);
+  const void* fn = nullptr;
+  int n_ctas = 0, cluster = 1;
+  size_t smem = 0;
+  if (T > kPairVocabLanesMax) {
+    const void* fn_pair = (const void*)head_pair_kernel<false, true>;
+    const int pair_tiles = (N + 2 * kBM - 1) / (2 * kBM);
+    const int n_groups = T > 2 * kPairRows ? 2 : 1;
+    int n_pairs = head_pair_slots(fn_pair);
+    if (n_groups == 2) n_pairs &= ~1;
+    if (n_pairs > 0) {
+      const int ks = pair_linear_ksplit(T, K, N, n_pairs);
+      if (n_pairs > pair_tiles * n_groups * ks) n_pairs = pair_tiles * n_groups * ks;
+      if (n_groups == 2) n_pairs &= ~1;
+      if (n_pairs > 0) {
+        ksplit = ks;
+        fn = fn_pair;
+        n_ctas = 2 * n_pairs;
+        cluster = 2;
+        smem = kPairSmemBytes;
+        a.n_tiles = pair_tiles;
+        a.ring_bytes = kPairRingBytes;
+        a.tmem_cols = 512;
+      }
+    }
+  }
+  if (!fn) {
+    fn = (const void*)head_tc_kernel<false, true>;
+    smem = head_smem_bytes(rows_alloc);
+    a.ring_bytes = head_ring_bytes(rows_alloc);
+    const int n_acc_alloc = 2 * rows_alloc <= 512 ? 2 : 1;
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(n_acc_alloc * rows_alloc)) cols <<= 1;
+    a.tmem_cols = cols;
+    const int slots = num_sms();
+    const int units = a.n_tiles * ksplit;
+    n_ctas = units < slots ? units : slots;
+  }
+  a.ksplit = ksplit;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(head_tc_kernel, linear)");
-  const int slots = num_sms();
-  const int units = a.n_tiles * ksplit;
-  const int n_ctas = units < slots ? units : slots;
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(linear kernel)");
   void* args[] = {(void*)&tw, (void*)&tx, (void*)&tx64, (void*)&tx128, (void*)&a};
   s = launch_pdl(fn, dim3(n_ctas), dim3(kHeadThreads), smem, st, args,
-                 "head_tc_kernel (linear) launch");
+                 cluster > 1 ? "head_pair_kernel (linear) launch" : "head_tc_kernel (linear) launch",
+                 cluster);
   if (s != SBD_OK || ksplit == 1) return s;
   const float* part = (const float*)ws;
   long long tn = (long long)T * N;

@@ -25,7 +25,12 @@ def _bf16(rng, shape, scale):
                                    (200, 256, 300), (256, 4096, 4096), (300, 128, 129),
                                    (512, 256, 1000),
                                    # few rows, narrow layers: K split over CTAs
-                                   (16, 4096, 4096), (2, 14336, 512), (64, 1024, 300)])
+                                   (16, 4096, 4096), (2, 14336, 512), (64, 1024, 300),
+                                   # above 192 rows: CTA pairs (one or two row
+                                   # groups; narrow layers with K ranges)
+                                   (193, 64, 1), (257, 128, 513), (384, 1024, 257),
+                                   (512, 4096, 6144), (512, 14336, 4096), (256, 14336, 512),
+                                   (320, 4096, 4096)])
 def test_matches_fp64_product(sbd, T, K, N):
     import torch
     rng = np.random.default_rng(T * 7 + N)
