@@ -211,7 +211,7 @@ sbd_status sbd_gumbel_philox(int32_t n_rows, const int32_t* row_ids, int32_t voc
  * bf16 (round to nearest even).  When a layer has too few output tiles to
  * fill the GPU, the in_features are cut into ranges whose fp32 partials go
  * through the workspace and are summed by a second kernel (the split is
- * chosen per call from the shape).  Above 192 rows the product runs on
+ * chosen per call from the shape).  Above 160 rows the product runs on
  * pairs of SMs (2-SM tensor-core MMAs).  All pointers 16-byte aligned,
  * caller-owned.  Asynchronous on `stream`.
  * Supported: dtype bf16, 0 <= rows <= 512, in_features a positive multiple

@@ -740,7 +740,7 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 // barriers; rank 0's thread issues the MMAs and commits them to the barriers
 // of both CTAs; the epilogue warps of rank 1 release an accumulator on rank
 // 0's barrier.  Two layouts, chosen from the live row count R:
-//  - Rows mode (R > kPairVocabLanesMax): the hidden rows are the A side
+//  - Rows mode (R > kPairVocabLanesMax = 160): the hidden rows are the A side
 //    (TMEM lane = hidden row, 128 per CTA) and W the B side (N = 256), so
 //    that each CTA's accumulator holds its rows' logits over all 256 ids of
 //    the tile.  Each epilogue thread owns one row and folds its logits into
@@ -756,13 +756,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 //    being fixed at 256 rows.
 // Measured on GB300: a 2-SM MMA of N = 256 takes ~65 ns, against ~95 ns for
 // the same work per SM as a 1-SM MMA, and each SM reads half of the hidden
-// rows from L2.  The column reductions over lanes took ~28 us per 256 x 128
-// logits, which bounds the vocabulary layout from ~200 rows; below that the
-// rows layout's fixed 256-row MMAs cost power (the kernel ran at ~1750 MHz
-// and ~950 W at 60 live rows, against 2070 MHz and ~450 W for
+// rows from L2.  The vocabulary layout's time grows with its padded N (131
+// live rows 192 us, 160 rows 198 us, 161-192 rows, padded to 192, 222 us)
+// while the rows layout takes ~212 us anywhere from 129 to 256 rows; below
+// that the rows layout's fixed 256-row MMAs also cost power (it ran at
+// ~1750 MHz and ~950 W at 60 live rows, against 2070 MHz and ~450 W for
 // head_tc_kernel) and lost to it.
 constexpr int kPairRows = 128;                 // hidden rows of one CTA per unit (M / 2)
-constexpr int kPairVocabLanesMax = 192;        // live rows up to which the vocabulary layout runs
+constexpr int kPairVocabLanesMax = 160;        // live rows up to which the vocabulary layout runs
 
 // One 16-column chunk of a row's logits z (vocabulary ids v0 .. v0 + 15, valid
 // below V) and Gumbel noise g folded into the running statistics.
@@ -890,9 +891,12 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int ring_bytes = a.ring_bytes - ep_bytes;
   const int h_box = rows_mode ? ((live_rows(grp * 2 * kPairRows) + 15) / 16 * 16) * kBK * 2
                               : (G / 2) * kBK * 2;
+  // (Vocabulary layout above N = 128: two stages, of longer W runs; at 131
+  // and 160 live rows 1-1.4 % faster than three.)
+  const int min_stages = !rows_mode && G > 128 ? 2 : 3;
   int boxes = kMaxBoxes;
-  while (boxes > 1 &&
-         ((a.H / kBK) % (boxes * ksplit) != 0 || ring_bytes / (boxes * (kABytes + h_box)) < 3))
+  while (boxes > 1 && ((a.H / kBK) % (boxes * ksplit) != 0 ||
+                       ring_bytes / (boxes * (kABytes + h_box)) < min_stages))
     boxes >>= 1;
   const int stage_bytes = boxes * (kABytes + h_box);
   int stages = ring_bytes / stage_bytes;

@@ -74,13 +74,14 @@ def test_bf16_shapes(sbd, B, k, V, H, tau):
     assert compare_head(d, "bf16", tau, ent, tok, with_noise=tau != 0.0) <= 1
 
 
-@pytest.mark.parametrize("R", [1, 17, 64, 80, 128, 144, 192, 193, 208, 255, 256, 257, 320, 400, 511,
+@pytest.mark.parametrize("R", [1, 17, 64, 80, 128, 129, 144, 160, 161, 192, 208, 255, 256, 257, 320, 400, 511,
                                512])
 def test_bf16_hidden_box_decomposition(sbd, R):
     """Exactly R masked rows out of 512 (the CTA-pair kernel): the live rows
     are loaded in boxes of 128, 64 and 16 rows (144 = 128 + 16,
-    208 = 128 + 64 + 16); up to 192 rows the vocabulary-lane layout, from
-    193 the row-lane layout, from 257 with two row groups; every row must
+    208 = 128 + 64 + 16); up to 160 rows the vocabulary-lane layout (above
+    128 rows with N = 160), from 161 the row-lane layout, from 257 with two
+    row groups; every row must
     come out right."""
     w = gen.shrink(gen.get_workload("llama8b_k16"), batch=16, block_k=32, vocab=1100, hidden=192,
                    cache_len=16)
@@ -102,6 +103,24 @@ def test_bf16_all_masked_and_none_masked(sbd):
     d["masked"] = np.zeros_like(d["masked"])
     ent, tok = run_head(sbd, d, "bf16", 1.0)
     assert np.isinf(ent).all() and (tok == -1).all()
+
+
+@pytest.mark.parametrize("philox", [False, True])
+def test_pair_kernel_without_masked_rows(sbd, philox):
+    """256 allocated rows (the CTA-pair kernel) and none masked: every CTA
+    pair allocates, meets and releases with no work, and every output is
+    +inf / -1."""
+    import torch
+    w = gen.shrink(gen.get_workload("llama8b_k16"), batch=16, block_k=16, vocab=3000, hidden=256)
+    d = step_inputs(w, seed=2)
+    hid, W = to_dev(d["hidden"], "bf16"), to_dev(d["w"], "bf16")
+    m = torch.zeros(16, 16, dtype=torch.uint8, device="cuda")
+    if philox:
+        ent, tok = sbd.sbd_head_entropy_sample_philox(hid, W, m, 5, 6, 1.0)
+    else:
+        ent, tok = sbd.sbd_head_entropy_sample(hid, W, m, torch.from_numpy(d["gumbel"]).cuda(), 1.0)
+    assert torch.isinf(ent).all() and (ent > 0).all() and (tok == -1).all()
+    assert sbd.sbd_device_error() == 0
 
 
 def test_bf16_uniform_and_one_hot_rows(sbd):

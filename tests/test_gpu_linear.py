@@ -26,9 +26,9 @@ def _bf16(rng, shape, scale):
                                    (512, 256, 1000),
                                    # few rows, narrow layers: K split over CTAs
                                    (16, 4096, 4096), (2, 14336, 512), (64, 1024, 300),
-                                   # above 192 rows: CTA pairs (one or two row
+                                   # above 160 rows: CTA pairs (one or two row
                                    # groups; narrow layers with K ranges)
-                                   (193, 64, 1), (257, 128, 513), (384, 1024, 257),
+                                   (161, 64, 1), (193, 64, 1), (257, 128, 513), (384, 1024, 257),
                                    (512, 4096, 6144), (512, 14336, 4096), (256, 14336, 512),
                                    (320, 4096, 4096)])
 def test_matches_fp64_product(sbd, T, K, N):
