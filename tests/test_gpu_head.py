@@ -105,6 +105,18 @@ def test_bf16_all_masked_and_none_masked(sbd):
     assert np.isinf(ent).all() and (tok == -1).all()
 
 
+@pytest.mark.parametrize("V", [1, 100, 128])
+def test_single_cta_kernel_for_one_vocabulary_tile(sbd, V):
+    """A vocabulary of one 128-row tile leaves no CTA pair: the single-CTA
+    kernel serves it."""
+    w = gen.shrink(gen.get_workload("llama8b_k16"), batch=3, block_k=8, vocab=V, hidden=256,
+                   decoded=("uniform", 0, 8))
+    d = step_inputs(w, seed=V)
+    for tau in (0.0, 1.0):
+        ent, tok = run_head(sbd, d, "bf16", tau, with_noise=tau != 0.0)
+        assert compare_head(d, "bf16", tau, ent, tok, with_noise=tau != 0.0) <= 1
+
+
 @pytest.mark.parametrize("philox", [False, True])
 def test_pair_kernel_without_masked_rows(sbd, philox):
     """256 allocated rows (the CTA-pair kernel) and none masked: every CTA
