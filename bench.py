@@ -252,15 +252,28 @@ def run_ours(args):
     step_inputs = ("q", "k_blk", "v_blk", "hidden") + (("gumbel",) if args.noise == "buffer" else ())
     eb_call = sbd.prepare_eb_select(ent, tok, gamma, masked, bt, n_un, stream=stream)
 
+    # The restore of the block state before each step (so that every timed
+    # step starts from the same masked positions) is harness, not method:
+    # it runs on a side stream beside the attention, which reads neither,
+    # and the LM head waits for it.
+    restore_stream = torch.cuda.Stream(dev)
+
     def step(ev=None):
         with torch.cuda.stream(stream):
-            masked.copy_(masked0, non_blocking=True)
-            bt.copy_(bt0, non_blocking=True)
+            fork = torch.cuda.Event()
+            fork.record(stream)
+            restore_stream.wait_event(fork)
+            with torch.cuda.stream(restore_stream):
+                masked.copy_(masked0, non_blocking=True)
+                bt.copy_(bt0, non_blocking=True)
+            restored = torch.cuda.Event()
+            restored.record(restore_stream)
             if ev is not None:
                 ev[0].record(stream)
             attn_call()
             if ev is not None:
                 ev[1].record(stream)
+            stream.wait_event(restored)
             head_call()
             if ev is not None:
                 ev[2].record(stream)
