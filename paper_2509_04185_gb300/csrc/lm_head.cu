@@ -6,27 +6,33 @@
 //   compact_rows_kernel  gathers the hidden rows of masked positions into a
 //                        dense [rows_alloc, H] buffer and a row map; writes
 //                        entropy = +inf / token = -1 for unmasked positions;
-//   head_tc_kernel       (bf16) persistent tcgen05 GEMM, swap-AB: 128 vocab
-//                        rows of W are the M side (A, K-major), the masked
-//                        hidden rows the N side (B, K-major).  A warp streams
-//                        W and hidden tiles into a shared-memory ring with
-//                        TMA; one thread issues tcgen05.mma into a
-//                        double-buffered fp32 accumulator in tensor memory;
-//                        eight epilogue warps (two per TMEM lane quadrant,
-//                        alternate 16-column chunks) read it back with
-//                        tcgen05.ld and reduce every logit column to running
+//   head_pair_kernel     (bf16) the LM head on CTA pairs (clusters of 2) with
+//                        2-SM tcgen05 MMAs of M = 256: W and the masked
+//                        hidden rows stream into shared-memory rings by TMA,
+//                        rank 0 issues the MMAs into double-buffered fp32
+//                        accumulators in tensor memory of both CTAs, and the
+//                        epilogue warps reduce every logit to running
 //                        statistics (max, sum of exponentials, entropy
-//                        numerator, best Gumbel score and id) -- logits never
-//                        reach HBM;
+//                        numerator, best Gumbel score and id) -- logits
+//                        never reach HBM.  Two layouts, chosen from the
+//                        live row count (see the kernel);
+//   head_tc_kernel       (bf16) the same on single CTAs with 1-SM MMAs,
+//                        swap-AB: 128 vocab rows of W are the M side (A,
+//                        K-major), the masked hidden rows the N side (B,
+//                        K-major); eight epilogue warps (two per TMEM lane
+//                        quadrant, alternate 16-column chunks) reduce each
+//                        logit column over the lanes.  The fallback where no
+//                        cluster of two fits or the vocabulary is one tile;
 //   head_f32_kernel      (fp32) the same reduction over exact fp32 FMAs;
 //   head_combine_kernel  merges the per-CTA statistics of each row into the
 //                        entropy (nats), the token and, when asked for, the
 //                        confidence max_v p_v = 1 / S.
 //
-// head_tc_kernel also serves sbd_linear (y = x W^T, a template switch): the
-// same main loop over all rows of x, an epilogue that stores the
-// accumulators (or, with K split over CTAs at few rows, fp32 partials that
-// linear_reduce_kernel sums).
+// Both tcgen05 kernels also serve sbd_linear (y = x W^T, a template
+// switch): the same main loop over all rows of x, an epilogue that stores
+// the outputs (or, with K split over CTAs, fp32 partials that
+// linear_reduce_kernel sums); head_tc_kernel up to 160 rows, the pair
+// kernel's rows layout above.
 #include <math.h>
 
 #include <mutex>
