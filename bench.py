@@ -839,7 +839,7 @@ def run_sweep(args):
                         "head": round(head_ms * 1000, 3), "eb_select": round(eb_ms * 1000, 3)},
         "roofline": {
             "kernel": "block attention, 32 layers (attn_tc_kernel up to 64 packed rows, "
-                      "attn_wide_kernel above, attn_bf16_kernel at 16 or fewer)",
+                      "attn_wide_kernel above)",
             "bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"],
             "peak_source": peak_src, "unit": "GB/s", "frac": round(attn_gbs / peaks["hbm_gbs"], 4),
             "traffic": sweep_traffic, "algorithmic_bytes": int(attn_bytes)},

@@ -1,10 +1,10 @@
 // Block attention on the tcgen05 tensor cores (arXiv 2509.04185, Eq. 5;
 // inference mask of Fig. 3) for bf16 inputs.
 //
-// Same partition as the mma.sync kernel -- one CTA per (KV split, KV head,
-// sequence), the G query heads of a KV head packed with the k block rows
-// into one row tile (row r = i*G + g, padded to 128) -- but both products run
-// on tcgen05 with their accumulators in tensor memory.  Keys stream in tiles
+// One CTA per (KV split, KV head, sequence), the G query heads of a KV head
+// packed with the k block rows into one row tile (row r = i*G + g, padded to
+// 128); both products run on tcgen05 with their accumulators in tensor
+// memory.  Keys stream in tiles
 // of 64 (one TMA stage each) and the products run on pairs of tiles:
 //
 //   S_q = Q K_q^T     A = Q (shared, K-major), B = the pair's K (shared,

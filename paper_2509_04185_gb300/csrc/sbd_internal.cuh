@@ -31,7 +31,7 @@ sbd_status encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dtype, uint32
 // Kernel launchers (each in the .cu file of its kernel).  Arguments were
 // validated by the API layer.
 struct AttnPlan {
-  int B, k, Hq, Hkv, G, D, Lmax, M, splits, stages, MT, KG;
+  int B, k, Hq, Hkv, G, D, Lmax, M, splits;
   bool order;         // CTAs take sequences longest first (more than one wave)
   bool cluster;       // the splits of a (sequence, KV head) merge in a cluster (tcgen05 path)
   int n_causal;       // block rows i < n_causal see block keys j <= i only

@@ -77,9 +77,9 @@ def test_f32(sbd, k, n_causal):
 
 
 @pytest.mark.parametrize("D", [64, 128])
-@pytest.mark.parametrize("G,k,n_causal", [(1, 16, 8), (2, 8, 4), (4, 4, 2),     # mma.sync kernel
-                                          (4, 8, 4), (3, 10, 5),                 # tcgen05, 4 copies
-                                          (4, 16, 8), (2, 32, 16),               # tcgen05, 2 copies
+@pytest.mark.parametrize("G,k,n_causal", [(1, 16, 8), (2, 8, 4), (4, 4, 2),     # <= 16 packed rows
+                                          (4, 8, 4), (3, 10, 5),
+                                          (4, 16, 8), (2, 32, 16),               # up to 64: attn_tc_kernel
                                           (4, 32, 16), (4, 32, 32), (8, 16, 1)])
 def test_bf16_kernels(sbd, D, G, k, n_causal):
     Hkv = 2
