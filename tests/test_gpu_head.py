@@ -193,3 +193,56 @@ def test_sweep_first_step(sbd, k):
                 exempt += 1
     print(f"token exemptions: {exempt} of {2 * B * k}")
     assert exempt <= 2
+
+
+@pytest.mark.parametrize("case", range(40))
+def test_pair_kernel_random_shapes(sbd, case):
+    """Seeded random shapes through the CTA-pair LM head: vocabularies that
+    leave a partial pair tile (or a pair tile past the end), hidden sizes of
+    any number of 64-column boxes, live-row counts across both layouts and
+    both row-group counts, noise from the buffer or in-kernel, tau 0 or 1."""
+    import torch
+    rng = np.random.default_rng(1000 + case)
+    B = int(rng.integers(1, 17))
+    k = int(rng.integers(1, 33))
+    while B * k > 512:
+        k //= 2
+    V = int(rng.integers(257, 6000))
+    H = 64 * int(rng.integers(1, 17))
+    R = int(rng.integers(0, B * k + 1))
+    tau = float(rng.choice([0.0, 1.0]))
+    philox = bool(rng.integers(0, 2)) and tau != 0.0
+    w = gen.shrink(gen.get_workload("llama8b_k16"), batch=B, block_k=k, vocab=V, hidden=H,
+                   cache_len=16)
+    d = step_inputs(w, seed=case)
+    m = np.zeros(B * k, dtype=np.uint8)
+    m[rng.choice(B * k, size=R, replace=False)] = 1
+    d["masked"] = m.reshape(B, k)
+    hid, W = to_dev(d["hidden"], "bf16"), to_dev(d["w"], "bf16")
+    mt = torch.from_numpy(d["masked"]).cuda()
+    if philox:
+        seed, offset = 77 + case, 5 * case
+        ent, tok = sbd.sbd_head_entropy_sample_philox(hid, W, mt, seed, offset, tau)
+        g, _ = oracle.philox_gumbel(np.arange(B * k), V, seed, offset)
+        d["gumbel"] = g.reshape(B, k, V)
+        slack = 2e-5 * tau
+    else:
+        g = torch.from_numpy(d["gumbel"]).cuda() if tau != 0.0 else None
+        ent, tok = sbd.sbd_head_entropy_sample(hid, W, mt, g, tau)
+        slack = 0.0
+    ent, tok = ent.cpu().numpy(), tok.cpu().numpy()
+    noise = d["gumbel"] if tau != 0.0 else None
+    rent, rtok, zs = oracle.head_entropy_sample(oracle.widen(d["hidden"], "bf16"), d["w"], "bf16",
+                                                d["masked"], noise, tau)
+    sel = d["masked"].astype(bool)
+    assert np.all(np.isinf(ent[~sel])) and np.all(tok[~sel] == -1)
+    if R:
+        assert np.abs(ent[sel] - rent[sel]).max() <= ENTROPY_TOL, (B, k, V, H, R)
+    exempt = 0
+    for (b, i), z in zs.items():
+        if tok[b, i] != rtok[b, i]:
+            gap = top2_gap(z, None if noise is None else noise[b, i], tau)
+            assert gap < token_tolerance(z, H // 16) + slack, (B, k, V, H, R, b, i, gap)
+            exempt += 1
+    assert exempt <= max(1, R // 50)
+    assert sbd.sbd_device_error() == 0

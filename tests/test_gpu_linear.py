@@ -55,3 +55,25 @@ def test_out_of_range_rows_are_not_written(sbd):
     big = torch.full((5, 200), 7.0, dtype=torch.bfloat16, device="cuda")
     sbd.sbd_linear(x, w, out=big[:3])
     assert torch.all(big[3:] == 7.0)
+
+
+@pytest.mark.parametrize("case", range(16))
+def test_random_shapes(sbd, case):
+    """Seeded random shapes on both sides of the CTA-pair threshold (160
+    rows): out_features that leave partial tiles, in_features of any number
+    of 64-column boxes (K split where the model picks one)."""
+    import torch
+    rng = np.random.default_rng(500 + case)
+    T = int(rng.integers(1, 513))
+    K = 64 * int(rng.integers(1, 65))
+    N = int(rng.integers(1, 3000))
+    xb, wb = _bf16(rng, (T, K), 1.0), _bf16(rng, (N, K), 0.02)
+    x = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
+    w = torch.from_numpy(wb.view(np.int16)).view(torch.bfloat16).cuda()
+    y = sbd.sbd_linear(x, w).float().cpu().numpy()
+    xf, wf = gen.bf16_bits_to_f32(xb), gen.bf16_bits_to_f32(wb)
+    ref = oracle.linear(xf, wf)
+    bound = np.abs(xf).astype(np.float64) @ np.abs(wf).astype(np.float64).T
+    tol = 2.0 ** -8 * np.abs(ref) + K * 2.0 ** -23 * bound + 1e-6
+    assert np.all(np.abs(y - ref) <= tol), (T, K, N, float(np.max(np.abs(y - ref) - tol)))
+    assert sbd.sbd_device_error() == 0
