@@ -295,12 +295,14 @@ __device__ __forceinline__ void cluster_merge(const TcArgs& a, int b, int hkv, u
 // warps sharing a row exchange their partial maxima through shared memory at
 // a named barrier and take identical decisions.
 //
-// PV with R = 2.  A tcgen05.mma of M = 128 and K = 16 measured the same time
-// for every N up to 256 (~95 ns on GB300), so N = D leaves half of each
-// instruction idle.  Each copy of a row therefore accumulates its own tile
-// only: lane r of P holds the row's probabilities over the keys of its
-// copy's tile, and one instruction with B = [V of 16 keys of tile 0 | V of
-// the same 16 rows of tile 1] (N = 2 D) adds P_copy0 V_tile0 to columns
+// PV with R = 2.  A tcgen05.mma of M = 128 and K = 16 costs nearly as much
+// at N = 128 as at N = 256 (47.6 against 65.4 ns of throughput on GB300),
+// and the MMAs lie on the chain S -> softmax -> P -> PV, so N = D would pay
+// almost a full instruction for half its work.  Each copy of a row
+// therefore accumulates its own tile only: lane r of P holds the row's
+// probabilities over the keys of its copy's tile, and one instruction with
+// B = [V of 16 keys of tile 0 | V of the same 16 rows of tile 1] (N = 2 D)
+// adds P_copy0 V_tile0 to columns
 // [0, D) and P_copy1 V_tile1 to columns [D, 2 D) of O (the other two blocks
 // of the product land in columns no lane reads).  4 instructions per pair
 // instead of 8; the two partial sums of a row are added in the epilogue.

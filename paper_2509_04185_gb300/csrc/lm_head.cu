@@ -760,9 +760,9 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 //    (N = R padded to 32, half of them in each CTA), with the column
 //    reductions over lanes.  The MMA's work then grows with R instead of
 //    being fixed at 256 rows.
-// Measured on GB300: a 2-SM MMA of N = 256 takes ~65 ns, against ~95 ns for
-// the same work per SM as a 1-SM MMA, and each SM reads half of the hidden
-// rows from L2.  The vocabulary layout's time grows with its padded N (131
+// Measured on GB300: a 2-SM MMA of N = 256 takes ~65 ns, the same rate per
+// SM as a 1-SM MMA; what the pair gains is that each SM reads half of the
+// hidden rows from L2 (the B operand is split between the two CTAs).  The vocabulary layout's time grows with its padded N (131
 // live rows 192 us, 160 rows 198 us, 161-192 rows, padded to 192, 222 us)
 // while the rows layout takes ~212 us anywhere from 129 to 256 rows; below
 // that the rows layout's fixed 256-row MMAs also cost power (it ran at
