@@ -447,6 +447,14 @@ def run_ours(args):
         e2e_steps(n_e2e, s2)
         e2.record(stream)
         torch.cuda.synchronize(dev)
+        if sbd.sbd_device_error() != 0:
+            raise RuntimeError("device error word set during the end-to-end steps")
+        # every step had the same inputs: the last step read back must match
+        # the device-timed steps' results
+        last = sets[(n_e2e - 1) % 2]["res"]
+        for k_, ref_ in (("tok", tok), ("n_un", n_un), ("masked", masked), ("bt", bt)):
+            if not torch.equal(last[k_], ref_.cpu()):
+                raise RuntimeError(f"end-to-end step read back a different {k_}")
         e2e_ms = max_over_ranks(s2.elapsed_time(e2), world, dev) / n_e2e
         e2e = {"value": round(job_us_per_step(e2e_ms, 1, world), 3), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
