@@ -532,13 +532,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
       // ------------------------------------------------ TMA producer
       if (lane == 0) {
         const uint64_t policy = l2_policy_evict_first();
-        int it = 0;
+        // the stage and its phase are counters, not quotients (see
+        // head_pair_kernel's producer)
+        int it = 0, s = 0;
+        uint32_t ph = 0;
         bool ok = true;
         for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
           const int tile = u / ksplit, kb0 = (u % ksplit) * num_kb;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % stages;
-            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&empty_bar[s], ph ^ 1, a.err)) {
               ok = false;
               break;
@@ -561,6 +562,10 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
                   tma_load_2d(hb + r0 * 128, &tmap_h64, &full_bar[s], col, r0);
               for (; r0 < n_eff; r0 += 16) tma_load_2d(hb + r0 * 128, &tmap_h, &full_bar[s], col, r0);
             }
+            if (++s == stages) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
         }
         // copies still in flight must land before the CTA exits
@@ -574,7 +579,8 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
         const int n_hi = n_eff > 256 ? n_eff - 256 : 0;
         const uint32_t idesc_lo = idesc_bf16_f32(kBM, n_eff > 256 ? 256 : n_eff);
         const uint32_t idesc_hi = idesc_bf16_f32(kBM, n_hi > 0 ? n_hi : 16);
-        int it = 0, local = 0;
+        int it = 0, local = 0, s = 0;
+        uint32_t ph = 0;
         bool ok = true;
         for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++local) {
           const int acc = n_acc == 2 ? (local & 1) : 0;
@@ -583,8 +589,6 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)acc * acc_stride;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % stages;
-            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&full_bar[s], ph, a.err)) {
               ok = false;
               break;
@@ -604,6 +608,10 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
               }
             }
             tc_commit(&empty_bar[s]);
+            if (++s == stages) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
           if (ok) tc_commit(&tmem_full[acc]);
         }
@@ -959,14 +967,19 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
         // W is read once: evict-first, except where two row groups share it
         const bool w_hint = n_groups == 1;
         const uint64_t policy = l2_policy_evict_first();
-        int it = 0;
+        // This thread shares an SM sub-partition with two busy epilogue warps
+        // and issues every copy, so its loop keeps little arithmetic per
+        // stage: the stage and its phase are counters, not quotients by the
+        // (run-time) stage count.  On GB300 that took the 60-row call from
+        // 174.5 to 166.6 us and the 512-row one 8 % down (same for the MMA
+        // thread below).
+        int it = 0, s = 0;
+        uint32_t ph = 0;
         bool ok = true;
         for (int tk = t_first; ok && tk < n_tk; tk += per_group) {
           const int t = tk / ksplit, kb0 = (tk % ksplit) * num_kb;
           const int w_row = (2 * t + rank) * kBM;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % stages;
-            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&empty_bar[s], ph ^ 1, a.err)) {
               ok = false;
               break;
@@ -991,6 +1004,10 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
               for (; r0 < h_count; r0 += 16)
                 tma_load_2d_pair(hb + r0 * 128, &tmap_h, fb, col, h_first + r0);
             }
+            if (++s == stages) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
         }
         // Copies still in flight must land before the CTA exits.  Rank 1
@@ -1007,7 +1024,8 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
         // rows mode: A = hidden rows, B = W (N = 256 vocabulary ids);
         // vocabulary mode: A = W, B = hidden rows (N = G)
         const uint32_t idesc = idesc_bf16_f32(2 * kPairRows, rows_mode ? 2 * kBM : G);
-        int it = 0, local = 0;
+        int it = 0, local = 0, s = 0;
+        uint32_t ph = 0;
         bool ok = true;
         for (int tk = t_first; ok && tk < n_tk; tk += per_group, ++local) {
           const int acc = local & 1;
@@ -1017,8 +1035,6 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)acc * 256u;
           for (int kb = 0; kb < num_kb; ++kb, ++it) {
-            const int s = it % stages;
-            const uint32_t ph = (it / stages) & 1;
             if (!mbar_wait(&full_bar[s], ph, a.err)) {
               ok = false;
               break;
@@ -1036,6 +1052,10 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
                                  (kb != 0 || x != 0 || kk != 0) ? 1u : 0u);
             }
             tc_commit_pair(&empty_bar[s], 0x3);
+            if (++s == stages) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
           if (ok) tc_commit_pair(&tmem_full[acc], 0x3);
         }
