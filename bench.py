@@ -710,6 +710,31 @@ class SweepLoop:
                 for s_ in range(k)]
         self.eb_call = sbd.prepare_eb_select(self.ent, self.tok, gamma, self.masked, self.bt,
                                              self.n_un, stream=stream)
+        self.graphs = []
+
+    def _graph_step(self, s_: int) -> None:
+        import torch
+        for c in self.attn_calls:
+            c()
+        self.head_calls[s_]()
+        self.eb_call()
+        self.left_h.copy_(self.masked.sum(dtype=torch.int32).view(1), non_blocking=True)
+
+    def capture(self) -> None:
+        """One CUDA graph per step index s = 0 .. k-1: every layer's
+        attention, the LM head of step s, the EB select and the 4-byte read
+        of the remaining masked count into pinned host memory.  block() then
+        launches one graph per step instead of each kernel from the host.
+        The loop's stream must not be the legacy default stream."""
+        import torch
+        graphs = []
+        with torch.cuda.stream(self.stream):
+            for s_ in range(self.w.block_k):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=self.stream):
+                    self._graph_step(s_)
+                graphs.append(g)
+        self.graphs = graphs
 
     def launches_per_step(self) -> int:
         """Kernels one step launches: per layer the attention kernel (+ the
@@ -726,10 +751,23 @@ class SweepLoop:
         import torch
         k = self.w.block_k
         stream = self.stream
+        graphed = bool(self.graphs) and ev is None and trace is None
+        with torch.cuda.stream(stream):
+            return self._block(k, stream, graphed, ev, trace)
+
+    def _block(self, k, stream, graphed, ev, trace) -> int:
+        import torch
         self.masked.fill_(1)
         self.bt.fill_(-1)
         steps = 0
         while True:
+            if graphed:
+                self.graphs[min(steps, k - 1)].replay()
+                stream.synchronize()
+                steps += 1
+                if int(self.left_h.item()) == 0 or steps >= k:
+                    return steps
+                continue
             if trace is not None:
                 stream.synchronize()
                 before = (self.masked.cpu().numpy(), self.bt.cpu().numpy())
@@ -776,16 +814,30 @@ def run_sweep(args):
     w = gen.get_workload(args.workload)
     B, k, Hq, Hkv, D, L = w.batch, w.block_k, w.n_q_heads, w.n_kv_heads, w.head_dim, w.max_cache_len
     V, H, NL = w.vocab, w.hidden, w.n_layers
-    stream = torch.cuda.current_stream(dev)
+    # a stream of its own: each step is replayed as a CUDA graph on it
+    stream = torch.cuda.Stream(dev)
+    torch.cuda.synchronize(dev)
     loop = SweepLoop(w, args.seed, args.noise, args.tau, args.gamma, dev, stream)
+    torch.cuda.synchronize(dev)
     block = loop.block
 
     sampler = ClockSampler(local_rank) if rank == 0 else None
     if sampler:
         sampler.start()
-    for _ in range(max(1, args.warmup // max(1, k // 2))):
+    n_warm = max(1, args.warmup // max(1, k // 2))
+    for _ in range(n_warm):
         block()
     torch.cuda.synchronize(dev)
+    graphed = False
+    if not args.no_graph:
+        try:
+            loop.capture()
+            block()
+            torch.cuda.synchronize(dev)
+            graphed = True
+        except Exception as ex:  # capture unsupported here: time the eager loop
+            print(f"sweep graph capture failed ({ex}); timing eager steps", file=sys.stderr)
+            loop.graphs = []
     if sbd.sbd_device_error() != 0:
         raise RuntimeError("device error word set during warm-up")
     if world > 1:
@@ -793,14 +845,13 @@ def run_sweep(args):
     torch.cuda.synchronize(dev)
     if sampler:
         sampler.mark("timed_start")
-    evs = []
     t0 = time.perf_counter()
     n_steps, n_blocks = 0, 0
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
     while n_steps < args.steps:
-        n_steps += block(evs)
+        n_steps += block()
         n_blocks += 1
     end.record(stream)
     torch.cuda.synchronize(dev)
@@ -808,6 +859,12 @@ def run_sweep(args):
     if sampler:
         sampler.mark("timed_end")
     total_ms = max_over_ranks(start.elapsed_time(end), world, dev)
+    # per-call durations: eager blocks with events between the calls, after
+    # the timed region
+    evs = []
+    for _ in range(2):
+        block(evs)
+    torch.cuda.synchronize(dev)
     attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     head_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     eb_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
@@ -853,6 +910,9 @@ def run_sweep(args):
             "traffic": sweep_traffic, "algorithmic_bytes": int(attn_bytes)},
         "head_first_step_bytes": int(head_bytes_first),
         "host_wall_s": round(wall, 3),
+        "step_launch": "one CUDA graph per step (every layer's attention, the LM head, the EB "
+                       "select, the 4-byte read of the remaining count)" if graphed
+                       else "eager launches",
         "clocks": clocks, "e2e": None, "cpu_baseline": None,
     }
     print(json.dumps(line), flush=True)

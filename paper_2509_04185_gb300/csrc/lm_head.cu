@@ -60,7 +60,10 @@ constexpr int kRingBytes = 216 * 1024;
 constexpr int kEpiWarps = 8;
 // Chunks of Gumbel noise an epilogue warp keeps in flight ahead of the one
 // it reduces (loads from HBM take longer than the reduction of one chunk).
-constexpr int kGAhead = 2;
+// Measured on GB300 with 2 to 6 chunks: 3 is best or within 0.5 us of it at
+// every row count (15 rows 156.6 -> 155.0 us against 2; 512 rows -6 %); 6
+// spills registers.
+constexpr int kGAhead = 3;
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kHeadThreads = 64 + kEpiThreads;   // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr float kLog2e = 1.4426950408889634f;
@@ -905,9 +908,10 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int ring_bytes = a.ring_bytes - ep_bytes;
   const int h_box = rows_mode ? ((live_rows(grp * 2 * kPairRows) + 15) / 16 * 16) * kBK * 2
                               : (G / 2) * kBK * 2;
-  // (Vocabulary layout above N = 128: two stages, of longer W runs; at 131
-  // and 160 live rows 1-1.4 % faster than three.)
-  const int min_stages = !rows_mode && G > 128 ? 2 : 3;
+  // At least three stages.  (Two stages of longer W runs had measured 1-1.4 %
+  // faster at 131 and 160 live rows while the control threads divided by
+  // the stage count; with counters three are 1.5-2 % faster there.)
+  const int min_stages = 3;
   int boxes = kMaxBoxes;
   while (boxes > 1 && ((a.H / kBK) % (boxes * ksplit) != 0 ||
                        ring_bytes / (boxes * (kABytes + h_box)) < min_stages))

@@ -139,3 +139,27 @@ def test_reduced_sweep_small_blocks(sbd):
         tok_ex, set_ex, o_steps = _replay(loop, trace, "buffer", 1.0, 0.1)
         assert o_steps == steps and tok_ex <= 1 and set_ex <= 1
         assert sbd.sbd_device_error() == 0
+
+
+@pytest.mark.parametrize("noise", ["buffer", "philox"])
+def test_graphed_sweep_loop_matches_eager(sbd, noise):
+    """The bench times the loop with one CUDA graph per step index; those
+    graphs take the same number of steps and commit the same tokens as the
+    eager loop (whose steps the test above replays through the oracle)."""
+    import torch
+
+    import bench
+    w = gen.shrink(gen.sweep_workload(16), n_layers=2, batch=2, cache_len=512, vocab=4096)
+    stream = torch.cuda.Stream()
+    loop = bench.SweepLoop(w, seed=5, noise=noise, tau=1.0, gamma=0.1,
+                           dev=torch.device("cuda"), stream=stream)
+    torch.cuda.synchronize()
+    eager_steps = loop.block()
+    bt_eager = loop.bt.cpu()
+    loop.capture()
+    for _ in range(2):
+        graph_steps = loop.block()
+        torch.cuda.synchronize()
+        assert graph_steps == eager_steps
+        assert torch.equal(loop.bt.cpu(), bt_eager)
+    assert sbd.sbd_device_error() == 0
