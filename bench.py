@@ -471,7 +471,9 @@ def run_ours(args):
     head_bytes = ab["head"]
     achieved = head_bytes / (head_ms * 1e-3) / 1e9
     kernel_file = os.path.join(ROOT, "paper_2509_04185_gb300", "csrc", "lm_head.cu")
-    traffic = profiled_traffic(args.workload, kernel_file)
+    # the committed captures read the noise from a buffer: no figure for the
+    # in-kernel noise variant
+    traffic = profiled_traffic(args.workload, kernel_file) if args.noise == "buffer" else None
     attn_gbs = ab["attention"] / (attn_ms * 1e-3) / 1e9
     step_bytes = ab["attention"] + ab["head"] + ab["eb"]
     ms_per_step = total_ms / args.steps
