@@ -1352,8 +1352,14 @@ head_pair_kernel(const __grid_constant__ CUtensorMap tmap_w,
 }
 
 // ------------------------------------------------------------ fp32 SIMT
-// One CTA per 128 vocab rows; z by sequential fp32 FMAs over H; the same
-// column statistics as the tensor-core epilogue.
+// One CTA per 128 vocab rows (thread = row) and the live hidden rows in
+// groups of 32.  W and the group's hidden rows pass through shared memory in
+// chunks of 32 columns, loaded coalesced, so each W element is read from
+// global memory once per group; each thread keeps its 32 logits in
+// registers.  Every logit is still the sequential fp32 FMA chain over H in
+// ascending order (padding columns add 0 * 0).  The same column statistics
+// as the tensor-core epilogue.
+constexpr int kF32Cols = 32;
 template <bool kPhilox>
 __global__ void __launch_bounds__(128)
 head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
@@ -1364,19 +1370,46 @@ head_f32_kernel(const float* __restrict__ hidden_c, const float* __restrict__ w,
   grid_dependency_wait();
   __shared__ float4 sm[4][32];
   __shared__ int si[4][32];
+  __shared__ float w_s[128][kF32Cols + 1];   // +1: rows land in distinct banks
+  __shared__ float h_s[32][kF32Cols];
   const int R = *n_rows;
-  const int v = blockIdx.x * 128 + threadIdx.x;
+  const int v0 = blockIdx.x * 128;
+  const int v = v0 + threadIdx.x;
   const bool valid = v < V;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool noisy = tau != 0.f && (kPhilox || gumbel != nullptr);
-  const float* wrow = w + (size_t)(valid ? v : 0) * H;
   for (int r0 = 0; r0 < R; r0 += 32) {
     const int nr = min(32, R - r0);
+    float zr[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) zr[j] = 0.f;
+    for (int c0 = 0; c0 < H; c0 += kF32Cols) {
+      const int nc = min(kF32Cols, H - c0);
+      __syncthreads();   // the previous chunk is consumed
+      for (int e = threadIdx.x; e < 128 * kF32Cols; e += 128) {
+        const int rr = e / kF32Cols, cc = e % kF32Cols;
+        w_s[rr][cc] = (v0 + rr < V && cc < nc) ? w[(size_t)(v0 + rr) * H + c0 + cc] : 0.f;
+      }
+      for (int e = threadIdx.x; e < 32 * kF32Cols; e += 128) {
+        const int jj = e / kF32Cols, cc = e % kF32Cols;
+        h_s[jj][cc] = (jj < nr && cc < nc) ? hidden_c[(size_t)(r0 + jj) * H + c0 + cc] : 0.f;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        if (j < nr) {
+          float acc = zr[j];
+#pragma unroll 8
+          for (int cc = 0; cc < kF32Cols; ++cc) acc = fmaf(h_s[j][cc], w_s[threadIdx.x][cc], acc);
+          zr[j] = acc;
+        }
+      }
+    }
     RowStats mine = rowstats_empty();
-    for (int j = 0; j < nr; ++j) {
-      const float* h = hidden_c + (size_t)(r0 + j) * H;
-      float z = 0.f;
-      for (int c = 0; c < H; ++c) z = fmaf(h[c], wrow[c], z);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      if (j >= nr) break;
+      const float z = zr[j];
       float g = 0.f;
       if (noisy && valid) {
         if constexpr (kPhilox) {
