@@ -92,6 +92,29 @@ def test_bf16_ragged_edges_every_kernel(sbd, k, splits):
     _run_and_compare(sbd, w, lens=[0, 1, 64, 65, 129], num_splits=splits)
 
 
+@pytest.mark.parametrize("case", range(24))
+def test_bf16_random_shapes(sbd, case):
+    """Seeded random shapes across both tcgen05 kernels (up to 64 and 65-128
+    packed rows G k), both head dims, ragged cache lengths (zero, tile
+    edges, anything up to the maximum) and automatic or explicit split
+    counts, so that both split merges (inside a cluster, and the combine
+    kernel) and empty splits are taken."""
+    rng = np.random.default_rng(1000 + case)
+    D = int(rng.choice([64, 128]))
+    Hkv = int(rng.integers(1, 5))
+    G = int(rng.integers(1, 9))
+    k = int(rng.integers(1, min(32, 128 // G) + 1))
+    B = int(rng.integers(1, 7))
+    Lmax = int(rng.integers(1, 1200))
+    lens = [int(x) for x in rng.integers(0, Lmax + 1, size=B)]
+    if case % 3 == 0:      # tile edges
+        lens[0] = min(Lmax, 64 * int(rng.integers(0, 4)) + int(rng.integers(0, 2)))
+    splits = int(rng.choice([0, 0, 0, 1, 2, 3, 5, 9, 17, 33]))
+    w = gen.shrink(BF16, batch=B, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv, head_dim=D,
+                   cache_len=(0, Lmax))
+    _run_and_compare(sbd, w, seed=case, num_splits=splits, lens=lens)
+
+
 def test_bf16_scale_override(sbd):
     w = gen.shrink(BF16, batch=1, block_k=4, n_q_heads=8, n_kv_heads=2, cache_len=100)
     _run_and_compare(sbd, w, scale=0.05)
