@@ -122,3 +122,24 @@ def test_append_overflow_is_reported_and_skipped(sbd):
     assert float(np.abs(got - ref).max()) <= BF16_ATTN_TOL
     assert np.array_equal(kc[1], d["k_cache"][1]) and np.array_equal(vc[1], d["v_cache"][1])
     assert np.array_equal(kc[0, 50:54], d["k_blk"][0, :4])
+
+
+@pytest.mark.parametrize("case", range(16))
+def test_bf16_random_shapes(sbd, case):
+    """Seeded random first-iteration calls: both tcgen05 kernels (up to 64
+    and 65-128 packed rows), both head dims, n_causal from 1 to k, ragged
+    lengths with room for the append, automatic or explicit split counts."""
+    rng = np.random.default_rng(2000 + case)
+    D = int(rng.choice([64, 128]))
+    Hkv = int(rng.integers(1, 4))
+    G = int(rng.integers(1, 9))
+    k = int(rng.integers(1, min(32, 128 // G) + 1))
+    n_causal = int(rng.integers(1, k + 1))
+    B = int(rng.integers(1, 5))
+    Lmax = int(rng.integers(n_causal, 900))
+    lens = [int(x) for x in rng.integers(0, Lmax - n_causal + 1, size=B)]
+    splits = int(rng.choice([0, 0, 1, 2, 5, 9]))
+    w = gen.shrink(BF16, batch=B, block_k=k, n_q_heads=G * Hkv, n_kv_heads=Hkv, head_dim=D,
+                   cache_len=(0, Lmax))
+    _check(sbd, w, _inputs(w, case, lens), n_causal, num_splits=splits)
+    assert sbd.sbd_device_error() == 0
