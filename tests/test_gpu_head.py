@@ -61,6 +61,24 @@ def test_tiny_f32_config(sbd):
             assert compare_head(d, w.dtype, tau, ent, tok, with_noise=tau != 0.0) == 0
 
 
+@pytest.mark.parametrize("case", range(12))
+def test_f32_random_shapes(sbd, case):
+    """Seeded random fp32 shapes through head_f32_kernel: hidden widths that
+    end in a partial 32-column chunk, partial vocabulary tiles, several
+    groups of 32 live rows, tau 0 and 1."""
+    rng = np.random.default_rng(3000 + case)
+    B = int(rng.integers(1, 5))
+    k = int(rng.integers(1, 33))
+    V = int(rng.integers(100, 2500))
+    H = int(rng.choice([4, 36, 64, 100, 260, 320]))
+    tau = float(rng.choice([0.0, 1.0]))
+    w = gen.shrink(gen.get_workload("tiny_f32"), batch=B, block_k=k, vocab=V, hidden=H,
+                   decoded=("uniform", 0, k))
+    d = step_inputs(w, seed=case)
+    ent, tok = run_head(sbd, d, "f32", tau, with_noise=tau != 0.0)
+    assert compare_head(d, "f32", tau, ent, tok, with_noise=tau != 0.0) <= 1
+
+
 @pytest.mark.parametrize("B,k,V,H", [(1, 1, 1000, 256), (1, 16, 4096 + 5, 512), (2, 16, 3000, 128),
                                      (3, 7, 777, 64), (16, 16, 2100, 256), (1, 17, 500, 128),
                                      (10, 30, 999, 64), (16, 32, 1500, 128),
