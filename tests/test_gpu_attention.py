@@ -60,6 +60,23 @@ def test_f32_shapes(sbd, k, Hq, Hkv):
 BF16 = gen.get_workload("llama8b_k16")
 
 
+@pytest.mark.parametrize("case", range(8))
+def test_f32_random_shapes(sbd, case):
+    """Seeded random fp32 shapes: both head dims, GQA groups, ragged cache
+    lengths (zero included) past the kernel's 128-key blocks."""
+    rng = np.random.default_rng(4000 + case)
+    D = int(rng.choice([64, 128]))
+    Hkv = int(rng.integers(1, 4))
+    G = int(rng.integers(1, 5))
+    k = int(rng.integers(1, 17))
+    B = int(rng.integers(1, 4))
+    Lmax = int(rng.integers(1, 400))
+    lens = [int(x) for x in rng.integers(0, Lmax + 1, size=B)]
+    w = gen.shrink(gen.get_workload("tiny_f32"), batch=B, block_k=k, n_q_heads=G * Hkv,
+                   n_kv_heads=Hkv, head_dim=D, cache_len=(0, Lmax))
+    _run_and_compare(sbd, w, seed=case, lens=lens)
+
+
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("G,k", [(4, 1), (4, 4), (1, 16), (4, 8), (3, 7), (2, 9), (4, 12), (4, 16),
                                  (2, 40 // 2), (4, 32), (8, 16), (3, 25), (5, 20), (2, 32)])
