@@ -773,12 +773,14 @@ head_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
 //    being fixed at 256 rows.
 // Measured on GB300: a 2-SM MMA of N = 256 takes ~65 ns, the same rate per
 // SM as a 1-SM MMA; what the pair gains is that each SM reads half of the
-// hidden rows from L2 (the B operand is split between the two CTAs).  The vocabulary layout's time grows with its padded N (131
-// live rows 192 us, 160 rows 198 us, 161-192 rows, padded to 192, 222 us)
-// while the rows layout takes ~212 us anywhere from 129 to 256 rows; below
-// that the rows layout's fixed 256-row MMAs also cost power (it ran at
-// ~1750 MHz and ~950 W at 60 live rows, against 2070 MHz and ~450 W for
-// head_tc_kernel) and lost to it.
+// hidden rows from L2 (the B operand is split between the two CTAs).  The
+// vocabulary layout's time grows with its padded N (when the threshold was
+// set: 131 live rows 192 us, 160 rows 198 us, 161-192 rows, padded to 192,
+// 222 us) while the rows layout took ~212 us anywhere from 129 to 256 rows;
+// re-checked on the current kernel, the rows layout is still slower at 131
+// rows (190.0 against 187.5 us).  Below that the rows layout's fixed
+// 256-row MMAs also cost power (it ran at ~1750 MHz and ~950 W at 60 live
+// rows, against 2070 MHz and ~450 W for head_tc_kernel) and lost to it.
 constexpr int kPairRows = 128;                 // hidden rows of one CTA per unit (M / 2)
 constexpr int kPairVocabLanesMax = 160;        // live rows up to which the vocabulary layout runs
 
